@@ -1,0 +1,180 @@
+/*
+ * regmem.h -- C ABI of the GB300 regulated streaming-attention library
+ * (libregmem.so).
+ *
+ * The library implements the per-frame, per-layer hot path of RegVGGT's
+ * streaming inference (arxiv 2609.23286):
+ *
+ *   1. temporal causal attention of the frame's queries over
+ *      [regulated KV memory ; the frame's own keys/values]      (Eq. 2, Eq. 3)
+ *   2. LSE-Saliency: per-key attention mass of a sampled query subset,
+ *      recovered from the rows' log-sum-exp                      (Sec. 3.3,
+ *      "FlashAttention-Compatible Saliency Estimation" and "Head-Specific
+ *      Token Retention")
+ *   3. per-head top-k admission of the most salient tokens into an append-only
+ *      HBM memory; the first frame is stored whole                (Eq. 4, Eq. 6)
+ *
+ * Conventions for every call
+ * --------------------------
+ * - Tensors named Q, K, V, out are bfloat16, row-major [N][H][64] (token,
+ *   head, channel), i.e. the usual [tokens, heads*head_dim] activation layout;
+ *   they are DEVICE pointers owned by the caller, 16-byte aligned.
+ * - Work is enqueued asynchronously on the stream given to
+ *   regmem_set_stream (default: the legacy default stream).  A call returns
+ *   before the GPU has finished.
+ * - Every call validates its arguments and the handle's state before
+ *   enqueueing anything: on any error it enqueues nothing, changes no state,
+ *   returns a negative regmem_status, and regmem_last_error() describes why.
+ *   Errors reported by the CUDA runtime are returned as REGMEM_ERR_CUDA.
+ *   Device-side bounded waits that expire are reported as REGMEM_ERR_TIMEOUT
+ *   by the next call (and by regmem_synchronize); the handle must then be
+ *   destroyed.
+ * - A handle is not thread-safe: one host thread at a time.
+ */
+#ifndef REGMEM_H
+#define REGMEM_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define REGMEM_API __attribute__((visibility("default")))
+#else
+#define REGMEM_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct regmem regmem_t; /* opaque; owns the per-layer HBM banks */
+
+typedef enum regmem_status {
+  REGMEM_OK = 0,
+  REGMEM_ERR_ARG = -1,         /* bad pointer, size, index or value          */
+  REGMEM_ERR_STATE = -2,       /* call out of order for the layer's state   */
+  REGMEM_ERR_CAPACITY = -3,    /* admission would overflow the bank          */
+  REGMEM_ERR_CUDA = -4,        /* CUDA runtime / driver error                */
+  REGMEM_ERR_UNSUPPORTED = -5, /* shape outside what the kernels handle      */
+  REGMEM_ERR_TIMEOUT = -6      /* a device-side bounded wait expired         */
+} regmem_status;
+
+/* Frame geometry.  Tokens of a frame are ordered [special tokens, patch tokens
+ * row-major over a grid_h x grid_w grid]; n_tokens = n_special + grid_h*grid_w
+ * (VGGT: 1 camera + 4 register tokens, then 37x37 patches of a 518x518 image
+ * at patch 14). */
+typedef struct regmem_frame_desc {
+  int32_t n_tokens;   /* N, tokens per frame (queries and keys of the frame)     */
+  int32_t n_special;  /* leading non-patch tokens                               */
+  int32_t grid_h;     /* patch rows                                             */
+  int32_t grid_w;     /* patch columns                                          */
+  int32_t ds;         /* query down-sampling window (Sec. 3.3: 2 = 2x2); 0 -> 2  */
+  int32_t max_frames; /* frames the banks must hold: capacity =
+                         N + (max_frames - 1) * budget rows per head and layer */
+  float scale;        /* softmax scale; 0 -> 1/sqrt(head_dim) (Eq. 2)            */
+  int32_t candidates; /* 0: only patch tokens may be admitted; 1: all tokens      */
+} regmem_frame_desc;
+
+/* Creates a handle for `layers` global-attention layers with `heads` heads of
+ * `head_dim` channels (head_dim must be 64), admitting at most `budget` rows
+ * per head per frame (Eq. 6: k = floor(gamma N); budget >= 0).  Allocates
+ * nothing on the GPU yet.  *out receives the handle (NULL on error). */
+REGMEM_API regmem_status regmem_create(regmem_t** out, int32_t layers, int32_t heads, int32_t head_dim,
+                            int32_t budget);
+
+/* Fixes the frame geometry and allocates, on the current CUDA device, the
+ * banks ([layers][heads][capacity][64] bf16 for K and for V, zero-filled) and
+ * the library's scratch.  Must be called once, before the first attend;
+ * ERR_STATE if called again. ERR_UNSUPPORTED if N exceeds 65536 or the
+ * number of admission candidates exceeds 8192. */
+REGMEM_API regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd);
+
+/* Stream (a cudaStream_t passed as void*) on which all later work is
+ * enqueued.  NULL selects the legacy default stream. */
+REGMEM_API regmem_status regmem_set_stream(regmem_t* h, void* stream);
+
+/* Eq. 3 for one layer and the current frame, fused with LSE-Saliency.
+ *   out[n][h][:] = softmax(Q_h K_h^T * scale) V_h over the keys
+ *                  [bank rows of (layer, h) ; the frame's N keys]
+ *   saliency[h][j] = sum over sampled queries i of exp(Z_ij - LSE_i),
+ *                  j in [0, N): the frame's keys; LSE_i is taken over every
+ *                  attended key, so saliency is the exact full-context
+ *                  attention mass (not renormalised over the frame).
+ * Q, K, V: device bf16 [N][H][64]; out: device bf16 [N][H][64];
+ * saliency: device fp32 [H][N].
+ * State: the layer must not have an attend pending (ERR_STATE).  K, V and
+ * saliency must stay valid and unmodified, in stream order, until this
+ * layer's regmem_admit has been enqueued; the library keeps the pointers. */
+REGMEM_API regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, const void* K,
+                                  const void* V, void* out, float* saliency);
+
+/* Same as regmem_attend_frame but with HOST buffers: Q, K, V and out are
+ * bf16 [N][H][64] and saliency fp32 [H][N] in host memory (pinned for
+ * asynchronous copies; pageable also works, synchronously).  K and V are
+ * staged into library-owned device buffers that stay valid until admit.
+ * The device->host copies of out and saliency are enqueued on the stream:
+ * they are complete after regmem_synchronize (or a sync of the stream). */
+REGMEM_API regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* hostQ,
+                                       const void* hostK, const void* hostV, void* hostOut,
+                                       float* hostSaliency);
+
+/* Eq. 4 / Eq. 6 for one layer, after its attend.
+ * - If the layer's memory is empty, the frame's N rows (all heads) become the
+ *   global anchor (Eq. 4) and k is ignored.
+ * - Otherwise, per head, the k candidate tokens with the largest saliency
+ *   (ties -> lower token index) are appended to that head's bank in ascending
+ *   token order (Eq. 6).  0 <= k <= min(budget, candidates) or ERR_ARG;
+ *   ERR_CAPACITY if the bank would overflow (nothing is appended).
+ * idx_out: optional device int32 [H][k] receiving the admitted token indices
+ * (ascending per head); NULL to skip.  On the anchor frame nothing is written.
+ * State: the layer must have an attend pending (ERR_STATE). */
+REGMEM_API regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out);
+
+/* Non-causal attention inside one frame (the frame-attention layers that
+ * alternate with the global ones, Sec. 3.1): out = softmax(Q K^T scale) V
+ * over the frame's own N keys, no memory, no saliency.  Uses the geometry of
+ * regmem_set_frame.  Layouts as in regmem_attend_frame. */
+REGMEM_API regmem_status regmem_frame_attention(regmem_t* h, const void* Q, const void* K, const void* V,
+                                     void* out);
+
+/* Empties every layer's memory (length 0, no attend pending); allocations
+ * and stream are kept.  Enqueues nothing. */
+REGMEM_API regmem_status regmem_reset(regmem_t* h);
+
+/* Rows currently held per head in `layer`'s bank (|M_t| of Eq. 6). */
+REGMEM_API regmem_status regmem_memory_len(const regmem_t* h, int32_t layer, int64_t* len);
+
+/* Rows each head's bank can hold (set by regmem_set_frame). */
+REGMEM_API regmem_status regmem_capacity(const regmem_t* h, int64_t* rows);
+
+/* Copies `layer`'s bank to host memory: hostK and hostV receive
+ * [H][len][64] bf16 with len = regmem_memory_len.  Synchronises the stream. */
+REGMEM_API regmem_status regmem_export_bank(regmem_t* h, int32_t layer, void* hostK, void* hostV);
+
+/* Replaces `layer`'s bank with host data [H][len][64] bf16 (checkpoint
+ * resume, or teacher forcing in tests).  len <= capacity; clears any pending
+ * attend.  Synchronises the stream. */
+REGMEM_API regmem_status regmem_import_bank(regmem_t* h, int32_t layer, const void* hostK,
+                                 const void* hostV, int64_t len);
+
+/* Enqueues a copy of the LSE rows of the most recent attend (any layer):
+ * dst is device fp32 [H][N] (natural log). */
+REGMEM_API regmem_status regmem_copy_lse(regmem_t* h, float* dst);
+
+/* Waits for all work enqueued on the handle's stream and reports any device
+ * status (REGMEM_ERR_TIMEOUT) or CUDA error. */
+REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
+
+/* Human-readable description of the last error on this handle ("" if none). */
+REGMEM_API const char* regmem_last_error(const regmem_t* h);
+
+/* Name of a status code. */
+REGMEM_API const char* regmem_status_string(regmem_status s);
+
+/* Frees every allocation of the handle (waits for its stream first). */
+REGMEM_API void regmem_destroy(regmem_t* h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* REGMEM_H */

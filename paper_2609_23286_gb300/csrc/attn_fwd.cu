@@ -1,0 +1,457 @@
+// Regulated causal attention with row log-sum-exp on the 5th-generation tensor
+// cores (Eq. 2 / Eq. 3, LSE of Sec. 3.3 "FlashAttention-Compatible Saliency
+// Estimation").
+//
+// For every head h and 128-row query tile the kernel computes
+//     O = softmax(Q K_c^T * scale) V_c,  LSE_i = log sum_j exp(Z_ij)
+// over K_c = [bank rows of head h (M of them) ; the frame's N keys], with no
+// mask inside the frame (frame-granular causality).  The key sequence is cut
+// into 128-row tiles: ceil(M/128) bank tiles followed by ceil(N/128) frame
+// tiles, each possibly ragged (columns past the valid count are masked).
+//
+// Work split (stream-K over the key dimension): the (unit, key tile) space,
+// unit = (head, query tile), is cut into `grid` contiguous equal ranges, one
+// per CTA.  A unit whose key tiles all fall in one CTA is finished there (O in
+// bf16 and LSE written directly); a unit cut between CTAs leaves normalised
+// fp32 partials (O_p, LSE_p) that attn_combine_kernel merges.
+//
+// CTA layout (128 threads = 4 warps, 2 CTAs per SM, so every SM sub-partition
+// holds two warps and each thread may use up to 255 registers):
+//   every thread owns one query row (TMEM lane): softmax on its S row,
+//   P -> TMEM, O rescale and epilogue.  Thread 0 additionally issues the TMA
+//   loads (prefetching two key tiles ahead through a 3-stage ring) and the
+//   tcgen05 MMAs.
+// TMEM (256 columns): S = Q K^T fp32 [0,128), P bf16 packed [128,192),
+// O fp32 [192,256).  Q K^T is an SS-MMA (both operands K-major in smem);
+// P V is a TS-MMA (P from TMEM, V MN-major in smem).  One mbarrier, committed
+// after each [P V of tile t ; Q K^T of tile t+1] pair, paces the loop: when it
+// completes, every MMA that read tile t-1's stage has finished, so that stage
+// is refilled with tile t+2.
+// The softmax keeps a stale running max and only rescales O when the max
+// grows by more than 2^8, so exp values stay <= 256.
+
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace regmem_dev {
+using namespace ptx;
+
+namespace {
+
+constexpr int BM = kTile, BN = kTile, HD = kHeadDim;
+constexpr int STAGES = 3;
+constexpr int TILE_BYTES = BM * HD * 2;  // 16 KB bf16 tile
+constexpr int THREADS = 128;
+constexpr uint32_t TMEM_COLS = 256, TM_S = 0, TM_P = 128, TM_O = 192;
+constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s: a hung pipeline gives up
+constexpr uint64_t DRAIN_NS = 200000000ull;   // 0.2 s for draining on abort
+constexpr float RESCALE_LOG2 = 8.0f;
+constexpr uint32_t IDESC_QK = idesc_bf16_f32(128, 128, false, false);
+constexpr uint32_t IDESC_PV = idesc_bf16_f32(128, 64, false, true);
+
+struct Smem {
+  uint8_t q[TILE_BYTES];
+  uint8_t k[STAGES][TILE_BYTES];
+  uint8_t v[STAGES][TILE_BYTES];
+  uint64_t q_full, k_full[STAGES], v_full[STAGES], mma_bar, fin_bar;
+  uint32_t tmem_base;
+  int abort_flag;
+  int never;  // always 0: abort word for waits that must not be cut short
+};
+// 7 tiles + 1 KB: two CTAs fill the SM's 228 KB exactly (1 KB reserved each).
+constexpr size_t SMEM_BYTES = 7 * TILE_BYTES + 1024;
+static_assert(sizeof(Smem) <= SMEM_BYTES, "smem layout");
+
+struct Params {
+  int N, H, M;
+  int nb, nkv, nqt;
+  long long total;
+  float scale_log2;
+  __nv_bfloat16* out;
+  float* lse;
+  float* part_o;
+  float* part_lse;
+  int* status;
+};
+
+__device__ __forceinline__ long long range_begin(int b, int G, long long T) {
+  return (long long)b * T / G;
+}
+
+__device__ __forceinline__ int tile_valid(const Params& p, int j) {
+  return j < p.nb ? min(BN, p.M - j * BN) : min(BN, p.N - (j - p.nb) * BN);
+}
+
+__device__ __forceinline__ void issue_qk(uint32_t d, uint32_t sq, uint32_t sk) {
+#pragma unroll
+  for (int kk = 0; kk < HD / 16; ++kk)
+    mma_ss(d, sdesc_sw128(sq + kk * 32), sdesc_sw128(sk + kk * 32), IDESC_QK, kk > 0);
+}
+
+// TMA loads of key tile x (global linear index over (unit, key tile)) into
+// ring stage st: K and V of bank rows or of the frame, 128 rows of one head.
+__device__ __forceinline__ void load_kv(Smem& sm, const Params& p, const CUtensorMap* tmK,
+                                        const CUtensorMap* tmV, const CUtensorMap* tmBK,
+                                        const CUtensorMap* tmBV, long long x, int st) {
+  const int u = (int)(x / p.nkv);
+  const int j = (int)(x - (long long)u * p.nkv);
+  const int h = u / p.nqt;
+  const uint32_t bk = smem_addr(&sm.k_full[st]), bv = smem_addr(&sm.v_full[st]);
+  mbar_arrive_expect_tx(bk, TILE_BYTES);
+  if (j < p.nb) tma_load_3d(smem_addr(sm.k[st]), tmBK, bk, 0, j * BN, h);
+  else tma_load_3d(smem_addr(sm.k[st]), tmK, bk, 0, h, (j - p.nb) * BN);
+  mbar_arrive_expect_tx(bv, TILE_BYTES);
+  if (j < p.nb) tma_load_3d(smem_addr(sm.v[st]), tmBV, bv, 0, j * BN, h);
+  else tma_load_3d(smem_addr(sm.v[st]), tmV, bv, 0, h, (j - p.nb) * BN);
+}
+
+__device__ __forceinline__ void load_q(Smem& sm, const Params& p, const CUtensorMap* tmQ, int u) {
+  const int h = u / p.nqt, qt = u - h * p.nqt;
+  mbar_arrive_expect_tx(smem_addr(&sm.q_full), TILE_BYTES);
+  tma_load_3d(smem_addr(sm.q), tmQ, smem_addr(&sm.q_full), 0, h, qt * BM);
+}
+
+__global__ void __launch_bounds__(THREADS, 2)
+    attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmBK,
+                    const __grid_constant__ CUtensorMap tmBV, const Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uintptr_t raw = reinterpret_cast<uintptr_t>(smem_raw);
+  const uintptr_t base = (raw + 1023) & ~uintptr_t(1023);
+  if (base + sizeof(Smem) > raw + SMEM_BYTES) {  // uniform for the whole CTA
+    if (threadIdx.x == 0) atomicOr(p.status, kStatusSmemAlign);
+    return;
+  }
+  Smem& sm = *reinterpret_cast<Smem*>(base);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  volatile int* abort_flag = &sm.abort_flag;
+  volatile int* never = &sm.never;
+  const bool issuer = (tid == 0);
+
+  const int G = gridDim.x, b = blockIdx.x;
+  const long long x_begin = range_begin(b, G, p.total), x_end = range_begin(b + 1, G, p.total);
+  const int nkv = p.nkv;
+  const int u_first = (int)(x_begin / nkv);
+  const uint32_t sq = smem_addr(sm.q);
+  const uint32_t b_qfull = smem_addr(&sm.q_full);
+  const uint32_t b_mma = smem_addr(&sm.mma_bar), b_fin = smem_addr(&sm.fin_bar);
+
+  // per-stage count of issued K/V loads and issued Q loads (issuer only)
+  int n_issued[STAGES] = {0, 0, 0};
+  int q_issued = 0;
+  if (issuer) {
+    sm.abort_flag = 0;
+    sm.never = 0;
+    mbar_init(b_qfull, 1);
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(smem_addr(&sm.k_full[s]), 1);
+      mbar_init(smem_addr(&sm.v_full[s]), 1);
+    }
+    mbar_init(b_mma, 1);
+    mbar_init(b_fin, 1);
+    fence_barrier_init();
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmK);
+    prefetch_tmap(&tmV);
+    prefetch_tmap(&tmBK);
+    prefetch_tmap(&tmBV);
+    load_q(sm, p, &tmQ, u_first);
+    ++q_issued;
+    for (int t = 0; t < STAGES - 1 && x_begin + t < x_end; ++t) {
+      load_kv(sm, p, &tmK, &tmV, &tmBK, &tmBV, x_begin + t, t);
+      ++n_issued[t];
+    }
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_addr(&sm.tmem_base), TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+
+  const int row = warp * 32 + lane;  // query row inside the tile = TMEM lane
+  const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
+  const float c = p.scale_log2;
+  int it = 0, piece = 0;             // it: tile counter inside this CTA's range
+  uint32_t mma_phase = 0;
+  bool stop = false;
+  for (long long x = x_begin; x < x_end && !stop;) {
+    const int u = (int)(x / nkv);
+    const int j0 = (int)(x - (long long)u * nkv);
+    const int j1 = (int)min((long long)nkv, j0 + (x_end - x));
+    const int h = u / p.nqt, qt = u - h * p.nqt;
+    const int n = j1 - j0;
+    if (issuer) {
+      bool ok = mbar_wait(b_qfull, piece & 1, abort_flag, WAIT_NS);
+      const int st = it % STAGES;
+      if (ok) ok = mbar_wait(smem_addr(&sm.k_full[st]), (it / STAGES) & 1, abort_flag, WAIT_NS);
+      if (ok) issue_qk(tmem + TM_S, sq, smem_addr(sm.k[st]));
+      mma_commit(b_mma);
+    }
+    float m_used = -INFINITY;  // running max of the logits, scaled to log2 units
+    float l = 0.f;             // running sum of exp2(z*c - m_used)
+    for (int jj = 0; jj < n; ++jj, ++it) {
+      const int j = j0 + jj;
+      const int st = it % STAGES;
+      const bool ok = mbar_wait(b_mma, mma_phase, abort_flag, WAIT_NS);
+      mma_phase ^= 1;
+      if (__syncthreads_or(!ok || *abort_flag)) {
+        stop = true;
+        break;
+      }
+      tc_fence_after();
+      if (issuer) {
+        // Q K^T of this tile and P V of the previous one are complete: refill
+        // the previous tile's stage two tiles ahead, and after the last
+        // Q K^T of this unit bring in the next unit's Q.
+        const long long xn = x_begin + it + (STAGES - 1);
+        if (xn < x_end) {
+          const int sn = (it + STAGES - 1) % STAGES;
+          load_kv(sm, p, &tmK, &tmV, &tmBK, &tmBV, xn, sn);
+          ++n_issued[sn];
+        }
+        if (jj == n - 1 && x + n < x_end) {
+          load_q(sm, p, &tmQ, u + 1);
+          ++q_issued;
+        }
+      }
+      uint32_t sr[128];
+      tmem_ld128(tmem + lane_off + TM_S, sr);
+      const int valid = tile_valid(p, j);
+      if (valid < BN) {
+#pragma unroll
+        for (int i = 0; i < 128; ++i)
+          if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
+      }
+      float mx8[8];
+#pragma unroll
+      for (int a = 0; a < 8; ++a) mx8[a] = __uint_as_float(sr[a]);
+#pragma unroll
+      for (int i = 8; i < 128; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(sr[i]));
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      const float mnew = mx * c;
+      float alpha = 1.f;
+      const bool need = mnew > m_used + RESCALE_LOG2;
+      if (need) {
+        alpha = ex2(m_used - mnew);  // 0 on the first tile (m_used = -inf)
+        l *= alpha;
+        m_used = mnew;
+      }
+      const float neg = -m_used;
+      uint32_t pk[64];
+      float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < 64; ++i) {
+        const float p0 = ex2(fmaf(__uint_as_float(sr[2 * i]), c, neg));
+        const float p1 = ex2(fmaf(__uint_as_float(sr[2 * i + 1]), c, neg));
+        ls[i & 3] += p0 + p1;
+        pk[i] = pack_bf16x2(p0, p1);
+      }
+      l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+      {
+        uint32_t (&pa)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pk[0]);
+        uint32_t (&pb)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pk[32]);
+        tmem_st32(tmem + lane_off + TM_P, pa);
+        tmem_st32(tmem + lane_off + TM_P + 32, pb);
+      }
+      if (jj > 0 && __any_sync(0xffffffffu, need)) {
+        // P V of the previous tile has completed (covered by the barrier just
+        // waited): rescale this warp's O rows in place.
+        uint32_t orr[64];
+        tmem_ld64(tmem + lane_off + TM_O, orr);
+#pragma unroll
+        for (int i = 0; i < 64; ++i) orr[i] = __float_as_uint(__uint_as_float(orr[i]) * alpha);
+        uint32_t (&oa)[32] = *reinterpret_cast<uint32_t(*)[32]>(&orr[0]);
+        uint32_t (&ob)[32] = *reinterpret_cast<uint32_t(*)[32]>(&orr[32]);
+        tmem_st32(tmem + lane_off + TM_O, oa);
+        tmem_st32(tmem + lane_off + TM_O + 32, ob);
+      }
+      tc_fence_before();
+      __syncthreads();
+      if (issuer) {
+        tc_fence_after();
+        const bool okv =
+            mbar_wait(smem_addr(&sm.v_full[st]), (it / STAGES) & 1, abort_flag, WAIT_NS);
+        if (okv) {
+          const uint32_t sv = smem_addr(sm.v[st]);
+#pragma unroll
+          for (int kk = 0; kk < BN / 16; ++kk)
+            mma_ts(tmem + TM_O, tmem + TM_P + kk * 8, sdesc_sw128(sv + kk * 2048), IDESC_PV,
+                   (jj > 0 || kk > 0) ? 1u : 0u);
+        }
+        if (jj + 1 < n) {
+          const int st2 = (it + 1) % STAGES;
+          const bool okk = okv && mbar_wait(smem_addr(&sm.k_full[st2]), ((it + 1) / STAGES) & 1,
+                                            abort_flag, WAIT_NS);
+          if (okk) issue_qk(tmem + TM_S, sq, smem_addr(sm.k[st2]));
+        }
+        mma_commit(b_mma);
+      }
+    }
+    if (stop) break;
+    // ------------------------------------------------------------ epilogue
+    const bool ok = mbar_wait(b_mma, mma_phase, abort_flag, WAIT_NS);
+    mma_phase ^= 1;
+    if (__syncthreads_or(!ok || *abort_flag)) {
+      stop = true;
+      break;
+    }
+    tc_fence_after();
+    uint32_t orr[64];
+    tmem_ld64(tmem + lane_off + TM_O, orr);
+    const float inv_l = 1.f / l;
+    const float lse_val = (m_used + __log2f(l)) * 0.69314718055994531f;
+    const int q = qt * BM + row;
+    if (j0 == 0 && j1 == nkv) {
+      if (q < p.N) {
+        uint4* dst = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + h) * HD);
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8) {
+          uint4 w;
+          w.x = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 0]) * inv_l, __uint_as_float(orr[c8 * 8 + 1]) * inv_l);
+          w.y = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 2]) * inv_l, __uint_as_float(orr[c8 * 8 + 3]) * inv_l);
+          w.z = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 4]) * inv_l, __uint_as_float(orr[c8 * 8 + 5]) * inv_l);
+          w.w = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 6]) * inv_l, __uint_as_float(orr[c8 * 8 + 7]) * inv_l);
+          dst[c8] = w;
+        }
+        p.lse[(size_t)h * p.N + q] = lse_val;
+      }
+    } else {
+      const int slot = (u == u_first) ? 0 : 1;
+      const size_t pr = ((size_t)b * 2 + slot) * BM + row;
+      float4* dst = reinterpret_cast<float4*>(p.part_o + pr * HD);
+#pragma unroll
+      for (int c4 = 0; c4 < 16; ++c4)
+        dst[c4] = make_float4(__uint_as_float(orr[c4 * 4 + 0]) * inv_l, __uint_as_float(orr[c4 * 4 + 1]) * inv_l,
+                              __uint_as_float(orr[c4 * 4 + 2]) * inv_l, __uint_as_float(orr[c4 * 4 + 3]) * inv_l);
+      p.part_lse[pr] = lse_val;
+    }
+    x += n;
+    ++piece;
+  }
+  if (issuer) {
+    // All MMAs issued have finished and every issued copy has landed before
+    // shared memory and TMEM are released (matters only after an abort).
+    mma_commit(b_fin);
+    mbar_wait(b_fin, 0, never, DRAIN_NS);
+    for (int s = 0; s < STAGES; ++s) {
+      if (n_issued[s] == 0) continue;
+      const uint32_t par = (uint32_t)((n_issued[s] - 1) & 1);
+      mbar_wait(smem_addr(&sm.k_full[s]), par, never, DRAIN_NS);
+      mbar_wait(smem_addr(&sm.v_full[s]), par, never, DRAIN_NS);
+    }
+    if (q_issued > 0) mbar_wait(b_qfull, (q_issued - 1) & 1, never, DRAIN_NS);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+  if (tid == 0 && sm.abort_flag) atomicOr(p.status, kStatusTimeout);
+}
+
+// Merges the partial (O_p, LSE_p) of every unit whose key tiles were split
+// across CTAs:  LSE = log sum_p exp(LSE_p),  O = sum_p exp(LSE_p - LSE) O_p.
+__global__ void __launch_bounds__(128) attn_combine_kernel(Params p, int G) {
+  const int u = blockIdx.x;
+  const long long T = p.total;
+  const int nkv = p.nkv;
+  auto cta_of = [&](long long x) {
+    long long bb = x * G / T;
+    while (bb + 1 < G && range_begin((int)bb + 1, G, T) <= x) ++bb;
+    while (bb > 0 && range_begin((int)bb, G, T) > x) --bb;
+    return (int)bb;
+  };
+  const int b_lo = cta_of((long long)u * nkv), b_hi = cta_of((long long)u * nkv + nkv - 1);
+  if (b_lo == b_hi) return;  // finished inside one CTA
+  const int h = u / p.nqt, qt = u - h * p.nqt;
+  const int row = threadIdx.x;
+  const int q = qt * BM + row;
+  if (q >= p.N) return;
+  float mx = -INFINITY;
+  for (int bb = b_lo; bb <= b_hi; ++bb) {
+    const int slot = (u == (int)(range_begin(bb, G, T) / nkv)) ? 0 : 1;
+    mx = fmaxf(mx, p.part_lse[((size_t)bb * 2 + slot) * BM + row]);
+  }
+  float den = 0.f;
+  for (int bb = b_lo; bb <= b_hi; ++bb) {
+    const int slot = (u == (int)(range_begin(bb, G, T) / nkv)) ? 0 : 1;
+    den += __expf(p.part_lse[((size_t)bb * 2 + slot) * BM + row] - mx);
+  }
+  const float lse = mx + __logf(den);
+  float acc[HD];
+#pragma unroll
+  for (int i = 0; i < HD; ++i) acc[i] = 0.f;
+  for (int bb = b_lo; bb <= b_hi; ++bb) {
+    const int slot = (u == (int)(range_begin(bb, G, T) / nkv)) ? 0 : 1;
+    const size_t pr = ((size_t)bb * 2 + slot) * BM + row;
+    const float w = __expf(p.part_lse[pr] - lse);
+    const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD);
+#pragma unroll
+    for (int c4 = 0; c4 < 16; ++c4) {
+      const float4 v = src[c4];
+      acc[c4 * 4 + 0] += w * v.x;
+      acc[c4 * 4 + 1] += w * v.y;
+      acc[c4 * 4 + 2] += w * v.z;
+      acc[c4 * 4 + 3] += w * v.w;
+    }
+  }
+  uint4* dst = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + h) * HD);
+#pragma unroll
+  for (int c8 = 0; c8 < 8; ++c8) {
+    uint4 w;
+    w.x = pack_bf16x2(acc[c8 * 8 + 0], acc[c8 * 8 + 1]);
+    w.y = pack_bf16x2(acc[c8 * 8 + 2], acc[c8 * 8 + 3]);
+    w.z = pack_bf16x2(acc[c8 * 8 + 4], acc[c8 * 8 + 5]);
+    w.w = pack_bf16x2(acc[c8 * 8 + 6], acc[c8 * 8 + 7]);
+    dst[c8] = w;
+  }
+  p.lse[(size_t)h * p.N + q] = lse;
+}
+
+}  // namespace
+
+cudaError_t attn_setup() {
+  cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attn_fwd_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+}
+
+int attn_ctas_per_sm() {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, attn_fwd_kernel, THREADS, SMEM_BYTES) !=
+      cudaSuccess)
+    return 1;
+  return n < 1 ? 1 : n;
+}
+
+cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s) {
+  Params p;
+  p.N = a.N;
+  p.H = a.H;
+  p.M = a.M;
+  p.nb = (a.M + BN - 1) / BN;
+  const int nf = (a.N + BN - 1) / BN;
+  p.nkv = p.nb + nf;
+  p.nqt = (a.N + BM - 1) / BM;
+  p.total = (long long)a.H * p.nqt * p.nkv;
+  p.scale_log2 = a.scale * 1.4426950408889634f;
+  p.out = a.out;
+  p.lse = a.lse;
+  p.part_o = a.part_o;
+  p.part_lse = a.part_lse;
+  p.status = a.status;
+  if (a.grid < 1 || (long long)a.grid > p.total) return cudaErrorInvalidValue;
+  attn_fwd_kernel<<<a.grid, THREADS, SMEM_BYTES, s>>>(*a.tmQ, *a.tmK, *a.tmV, *a.tmBK, *a.tmBV, p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || !combine) return e;
+  attn_combine_kernel<<<a.H * p.nqt, 128, 0, s>>>(p, a.grid);
+  return cudaGetLastError();
+}
+
+}  // namespace regmem_dev

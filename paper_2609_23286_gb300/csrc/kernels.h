@@ -1,0 +1,81 @@
+// Internal launch interface between the C-ABI layer (regmem_api.cu) and the
+// kernels.  Nothing here is exported from the shared library.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+namespace regmem_dev {
+
+constexpr int kHeadDim = 64;    // channels per head handled by the kernels
+constexpr int kTile = 128;      // query rows / key rows per tile
+
+// Bits of the device status word (written by kernels, read by the host).
+constexpr int kStatusTimeout = 1;    // a bounded wait expired
+constexpr int kStatusSmemAlign = 2;  // dynamic shared memory not 1 KB aligned
+
+// Attention over [bank rows ; frame rows] for every (head, 128-row query tile).
+struct AttnArgs {
+  const CUtensorMap* tmQ;   // frame tensors [N][H][64] bf16, box 64x1x128
+  const CUtensorMap* tmK;
+  const CUtensorMap* tmV;
+  const CUtensorMap* tmBK;  // bank [H][cap][64] bf16, box 64x128x1
+  const CUtensorMap* tmBV;
+  int N, H, M;              // frame tokens, heads, bank rows per head
+  float scale;
+  __nv_bfloat16* out;       // [N][H][64]
+  float* lse;               // [H][N]
+  float* part_o;            // [grid][2][128][64] split-piece partial outputs
+  float* part_lse;          // [grid][2][128]
+  int* status;
+  int grid;                 // CTAs of the attention kernel (<= H*nqt*nkv)
+};
+
+// Scratch sizes for a given grid.
+inline size_t attn_part_o_floats(int grid) { return (size_t)grid * 2 * kTile * kHeadDim; }
+inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kTile; }
+
+cudaError_t attn_setup();                              // kernel attributes (once)
+int attn_ctas_per_sm();                                // resident CTAs per SM
+// `combine`: some unit's key range is cut between CTAs, so the partials must
+// be merged (decided on the host from the same schedule formula).
+cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s);
+
+// LSE-Saliency over the frame's own keys, per (head, 128-key tile).
+struct SalArgs {
+  const CUtensorMap* tmK;   // frame K map (same as the attention's)
+  const __nv_bfloat16* Q;   // [N][H][64]
+  const int* qidx;          // sampled query tokens, [nq]
+  int nq;
+  const float* lse;         // [H][N]
+  int N, H;
+  float scale;
+  float* sal;               // [H][N]
+  int* status;
+};
+cudaError_t saliency_setup();
+cudaError_t launch_saliency(const SalArgs& a, cudaStream_t s);
+
+// Per-head top-k of the candidates' saliency and append to the bank.
+struct AdmitArgs {
+  const float* sal;         // [H][N]
+  const __nv_bfloat16* K;   // [N][H][64]
+  const __nv_bfloat16* V;
+  __nv_bfloat16* bankK;     // this layer's bank [H][cap][64]
+  __nv_bfloat16* bankV;
+  long long cap;
+  long long M;              // rows already in the bank
+  int N, H, cand_lo, k;
+  int32_t* idx_out;         // optional [H][k]
+};
+cudaError_t admit_setup();
+cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s);
+// First frame (Eq. 4): bank[h][0:N] = frame rows of head h.
+cudaError_t launch_anchor(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
+                          __nv_bfloat16* bankV, long long cap, int N, int H, cudaStream_t s);
+
+constexpr int kMaxCandidates = 8192;
+
+}  // namespace regmem_dev

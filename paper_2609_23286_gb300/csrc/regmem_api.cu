@@ -1,0 +1,530 @@
+// C ABI of libregmem.so (declared in include/regmem.h): handle, argument and
+// state validation, HBM bank ownership, TMA descriptor set-up and kernel
+// launches.  Every compute step runs in this library's kernels.
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "kernels.h"
+#include "regmem.h"
+
+using namespace regmem_dev;
+
+struct regmem {
+  int layers = 0, heads = 0, head_dim = 0, budget = 0;
+  bool frame_set = false;
+  int device = 0;
+  int N = 0, n_special = 0, grid_h = 0, grid_w = 0, ds = 2, cand_lo = 0, nq = 0;
+  int max_frames = 0;
+  float scale = 0.f;
+  long long cap = 0;
+  cudaStream_t stream = nullptr;
+
+  std::vector<long long> len;
+  std::vector<int> pending;
+  std::vector<const __nv_bfloat16*> pK, pV;
+  std::vector<float*> pS;
+
+  __nv_bfloat16* bankK = nullptr;  // [layers][H][cap][64]
+  __nv_bfloat16* bankV = nullptr;
+  std::vector<CUtensorMap> tmBK, tmBV;
+
+  float* lse = nullptr;       // [H][N]
+  int* qidx = nullptr;        // [nq]
+  float* part_o = nullptr;    // split-KV partials
+  float* part_lse = nullptr;
+  int attn_grid = 0;
+  int* status_host = nullptr; // mapped pinned word written by kernels
+  int* status_dev = nullptr;
+
+  // staging for the host-buffer entry point (allocated on first use)
+  __nv_bfloat16* stQ = nullptr;
+  __nv_bfloat16* stOut = nullptr;
+  float* stSal = nullptr;
+  std::vector<__nv_bfloat16*> stK, stV;
+
+  std::string err;
+};
+
+namespace {
+
+regmem_status fail(regmem_t* h, regmem_status s, const char* fmt, ...) {
+  if (h) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    h->err = buf;
+  }
+  return s;
+}
+
+regmem_status cuda_fail(regmem_t* h, cudaError_t e, const char* what) {
+  return fail(h, REGMEM_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define RM_CUDA(h, call)                                  \
+  do {                                                    \
+    cudaError_t e_ = (call);                              \
+    if (e_ != cudaSuccess) return cuda_fail((h), e_, #call); \
+  } while (0)
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// Frame tensor [N][H][64] bf16 viewed as 3-D (channel, head, token); one box is
+// one head's 128 consecutive tokens, 128-byte swizzled.
+bool encode_frame_map(CUtensorMap* m, const void* ptr, int N, int H) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)H, (cuuint64_t)N};
+  cuuint64_t strides[2] = {(cuuint64_t)kHeadDim * 2, (cuuint64_t)H * kHeadDim * 2};
+  cuuint32_t box[3] = {(cuuint32_t)kHeadDim, 1, (cuuint32_t)kTile};
+  cuuint32_t es[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Bank [H][cap][64] bf16 viewed as 3-D (channel, row, head); one box is 128
+// rows of one head.
+bool encode_bank_map(CUtensorMap* m, const void* ptr, long long cap, int H) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)cap, (cuuint64_t)H};
+  cuuint64_t strides[2] = {(cuuint64_t)kHeadDim * 2, (cuuint64_t)cap * kHeadDim * 2};
+  cuuint32_t box[3] = {(cuuint32_t)kHeadDim, (cuuint32_t)kTile, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+regmem_status check_device_status(regmem_t* h) {
+  if (h->status_host && *reinterpret_cast<volatile int*>(h->status_host) != 0) {
+    const int s = *reinterpret_cast<volatile int*>(h->status_host);
+    return fail(h, REGMEM_ERR_TIMEOUT,
+                "a kernel reported device status 0x%x (%s); destroy the handle", s,
+                (s & kStatusTimeout) ? "bounded wait expired" : "shared-memory alignment");
+  }
+  return REGMEM_OK;
+}
+
+regmem_status ready(regmem_t* h, int layer, bool need_layer) {
+  if (!h) return REGMEM_ERR_ARG;
+  if (!h->frame_set) return fail(h, REGMEM_ERR_STATE, "regmem_set_frame has not been called");
+  if (need_layer && (layer < 0 || layer >= h->layers))
+    return fail(h, REGMEM_ERR_ARG, "layer %d out of range [0, %d)", layer, h->layers);
+  regmem_status s = check_device_status(h);
+  if (s != REGMEM_OK) return s;
+  if (cudaSetDevice(h->device) != cudaSuccess)
+    return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
+  return REGMEM_OK;
+}
+
+// Is any (head, query tile) unit's key range cut between two CTAs?
+bool any_split(long long units, long long nkv, long long G) {
+  const long long T = units * nkv;
+  auto begin = [&](long long b) { return b * T / G; };
+  auto cta_of = [&](long long x) {
+    long long b = x * G / T;
+    while (b + 1 < G && begin(b + 1) <= x) ++b;
+    while (b > 0 && begin(b) > x) --b;
+    return b;
+  };
+  for (long long u = 0; u < units; ++u)
+    if (cta_of(u * nkv) != cta_of(u * nkv + nkv - 1)) return true;
+  return false;
+}
+
+regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K, const void* V,
+                            void* out, int M) {
+  CUtensorMap tq, tk, tv;
+  if (!encode_frame_map(&tq, Q, h->N, h->heads) || !encode_frame_map(&tk, K, h->N, h->heads) ||
+      !encode_frame_map(&tv, V, h->N, h->heads))
+    return fail(h, REGMEM_ERR_CUDA, "cuTensorMapEncodeTiled failed for the frame tensors");
+  AttnArgs a;
+  a.tmQ = &tq;
+  a.tmK = &tk;
+  a.tmV = &tv;
+  a.tmBK = &h->tmBK[layer];
+  a.tmBV = &h->tmBV[layer];
+  a.N = h->N;
+  a.H = h->heads;
+  a.M = M;
+  a.scale = h->scale;
+  a.out = static_cast<__nv_bfloat16*>(out);
+  a.lse = h->lse;
+  a.part_o = h->part_o;
+  a.part_lse = h->part_lse;
+  a.status = h->status_dev;
+  a.grid = h->attn_grid;
+  const long long nqt = (h->N + kTile - 1) / kTile;
+  const long long nkv = (M + kTile - 1) / kTile + nqt;
+  const long long T = (long long)h->heads * nqt * nkv;
+  const long long G = T < a.grid ? T : a.grid;
+  a.grid = (int)G;
+  RM_CUDA(h, launch_attention(a, any_split((long long)h->heads * nqt, nkv, G), h->stream));
+  return REGMEM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* regmem_status_string(regmem_status s) {
+  switch (s) {
+    case REGMEM_OK: return "REGMEM_OK";
+    case REGMEM_ERR_ARG: return "REGMEM_ERR_ARG";
+    case REGMEM_ERR_STATE: return "REGMEM_ERR_STATE";
+    case REGMEM_ERR_CAPACITY: return "REGMEM_ERR_CAPACITY";
+    case REGMEM_ERR_CUDA: return "REGMEM_ERR_CUDA";
+    case REGMEM_ERR_UNSUPPORTED: return "REGMEM_ERR_UNSUPPORTED";
+    case REGMEM_ERR_TIMEOUT: return "REGMEM_ERR_TIMEOUT";
+  }
+  return "REGMEM_UNKNOWN";
+}
+
+const char* regmem_last_error(const regmem_t* h) { return h ? h->err.c_str() : "null handle"; }
+
+regmem_status regmem_create(regmem_t** out, int32_t layers, int32_t heads, int32_t head_dim,
+                            int32_t budget) {
+  if (!out) return REGMEM_ERR_ARG;
+  *out = nullptr;
+  if (layers < 1 || heads < 1 || budget < 0) return REGMEM_ERR_ARG;
+  if (head_dim != kHeadDim) return REGMEM_ERR_UNSUPPORTED;
+  regmem_t* h = new (std::nothrow) regmem_t();
+  if (!h) return REGMEM_ERR_ARG;
+  h->layers = layers;
+  h->heads = heads;
+  h->head_dim = head_dim;
+  h->budget = budget;
+  h->len.assign(layers, 0);
+  h->pending.assign(layers, 0);
+  h->pK.assign(layers, nullptr);
+  h->pV.assign(layers, nullptr);
+  h->pS.assign(layers, nullptr);
+  h->stK.assign(layers, nullptr);
+  h->stV.assign(layers, nullptr);
+  *out = h;
+  return REGMEM_OK;
+}
+
+regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
+  if (!h || !fd) return REGMEM_ERR_ARG;
+  if (h->frame_set) return fail(h, REGMEM_ERR_STATE, "frame geometry already set");
+  const int ds = fd->ds == 0 ? 2 : fd->ds;
+  if (fd->n_special < 0 || fd->grid_h < 1 || fd->grid_w < 1 || ds < 1 || fd->max_frames < 1 ||
+      fd->n_tokens != fd->n_special + fd->grid_h * fd->grid_w || fd->scale < 0.f ||
+      !std::isfinite(fd->scale) || (fd->candidates != 0 && fd->candidates != 1))
+    return fail(h, REGMEM_ERR_ARG, "inconsistent frame descriptor");
+  const int N = fd->n_tokens;
+  if (N > 65536) return fail(h, REGMEM_ERR_UNSUPPORTED, "n_tokens %d > 65536", N);
+  const int cand_lo = fd->candidates == 0 ? fd->n_special : 0;
+  if (N - cand_lo > kMaxCandidates)
+    return fail(h, REGMEM_ERR_UNSUPPORTED, "%d admission candidates > %d", N - cand_lo,
+                kMaxCandidates);
+  // sampled queries: top-left of each ds x ds window of the patch grid
+  std::vector<int> q;
+  for (int r = 0; r < fd->grid_h; r += ds)
+    for (int c = 0; c < fd->grid_w; c += ds) q.push_back(fd->n_special + r * fd->grid_w + c);
+  if ((int)q.size() > 8192) return fail(h, REGMEM_ERR_UNSUPPORTED, "too many sampled queries");
+  const long long cap = (long long)N + (long long)(fd->max_frames - 1) * h->budget;
+  if (cap > (1LL << 31) - 1) return fail(h, REGMEM_ERR_UNSUPPORTED, "bank capacity too large");
+
+  RM_CUDA(h, cudaGetDevice(&h->device));
+  int sms = 0;
+  RM_CUDA(h, cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, h->device));
+  RM_CUDA(h, attn_setup());
+  RM_CUDA(h, saliency_setup());
+  RM_CUDA(h, admit_setup());
+  if (!encode_fn()) return fail(h, REGMEM_ERR_CUDA, "cuTensorMapEncodeTiled entry point missing");
+
+  const size_t bank_elems = (size_t)h->layers * h->heads * cap * kHeadDim;
+  h->attn_grid = sms * attn_ctas_per_sm();
+  RM_CUDA(h, cudaMalloc(&h->bankK, bank_elems * 2));
+  RM_CUDA(h, cudaMalloc(&h->bankV, bank_elems * 2));
+  RM_CUDA(h, cudaMemset(h->bankK, 0, bank_elems * 2));
+  RM_CUDA(h, cudaMemset(h->bankV, 0, bank_elems * 2));
+  RM_CUDA(h, cudaMalloc(&h->lse, (size_t)h->heads * N * sizeof(float)));
+  RM_CUDA(h, cudaMalloc(&h->qidx, q.size() * sizeof(int) + 4));
+  RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
+  RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_floats(h->attn_grid) * sizeof(float)));
+  RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid) * sizeof(float)));
+  RM_CUDA(h, cudaHostAlloc(&h->status_host, sizeof(int), cudaHostAllocMapped));
+  *h->status_host = 0;
+  RM_CUDA(h, cudaHostGetDevicePointer(&h->status_dev, h->status_host, 0));
+
+  h->tmBK.resize(h->layers);
+  h->tmBV.resize(h->layers);
+  for (int l = 0; l < h->layers; ++l) {
+    const size_t off = (size_t)l * h->heads * cap * kHeadDim;
+    if (!encode_bank_map(&h->tmBK[l], h->bankK + off, cap, h->heads) ||
+        !encode_bank_map(&h->tmBV[l], h->bankV + off, cap, h->heads))
+      return fail(h, REGMEM_ERR_CUDA, "cuTensorMapEncodeTiled failed for the bank");
+  }
+  h->N = N;
+  h->n_special = fd->n_special;
+  h->grid_h = fd->grid_h;
+  h->grid_w = fd->grid_w;
+  h->ds = ds;
+  h->cand_lo = cand_lo;
+  h->nq = (int)q.size();
+  h->max_frames = fd->max_frames;
+  h->scale = fd->scale == 0.f ? 1.f / std::sqrt((float)h->head_dim) : fd->scale;
+  h->cap = cap;
+  h->frame_set = true;
+  return REGMEM_OK;
+}
+
+regmem_status regmem_set_stream(regmem_t* h, void* stream) {
+  if (!h) return REGMEM_ERR_ARG;
+  h->stream = static_cast<cudaStream_t>(stream);
+  return REGMEM_OK;
+}
+
+regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, const void* K,
+                                  const void* V, void* out, float* saliency) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if (!Q || !K || !V || !out || !saliency)
+    return fail(h, REGMEM_ERR_ARG, "null tensor pointer");
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(out) || !aligned16(saliency))
+    return fail(h, REGMEM_ERR_ARG, "tensor pointers must be 16-byte aligned");
+  if (h->pending[layer])
+    return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
+                layer);
+  const long long M = h->len[layer];
+  s = run_attention(h, layer, Q, K, V, out, (int)M);
+  if (s != REGMEM_OK) return s;
+  CUtensorMap tk;
+  if (!encode_frame_map(&tk, K, h->N, h->heads))
+    return fail(h, REGMEM_ERR_CUDA, "cuTensorMapEncodeTiled failed for K");
+  SalArgs sa;
+  sa.tmK = &tk;
+  sa.Q = static_cast<const __nv_bfloat16*>(Q);
+  sa.qidx = h->qidx;
+  sa.nq = h->nq;
+  sa.lse = h->lse;
+  sa.N = h->N;
+  sa.H = h->heads;
+  sa.scale = h->scale;
+  sa.sal = saliency;
+  sa.status = h->status_dev;
+  RM_CUDA(h, launch_saliency(sa, h->stream));
+  h->pending[layer] = 1;
+  h->pK[layer] = static_cast<const __nv_bfloat16*>(K);
+  h->pV[layer] = static_cast<const __nv_bfloat16*>(V);
+  h->pS[layer] = saliency;
+  return REGMEM_OK;
+}
+
+regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* hostQ,
+                                       const void* hostK, const void* hostV, void* hostOut,
+                                       float* hostSaliency) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if (!hostQ || !hostK || !hostV || !hostOut || !hostSaliency)
+    return fail(h, REGMEM_ERR_ARG, "null host pointer");
+  if (h->pending[layer])
+    return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
+                layer);
+  const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
+  const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
+  if (!h->stQ) {
+    RM_CUDA(h, cudaMalloc(&h->stQ, tbytes));
+    RM_CUDA(h, cudaMalloc(&h->stOut, tbytes));
+    RM_CUDA(h, cudaMalloc(&h->stSal, sbytes));
+  }
+  if (!h->stK[layer]) {
+    RM_CUDA(h, cudaMalloc(&h->stK[layer], tbytes));
+    RM_CUDA(h, cudaMalloc(&h->stV[layer], tbytes));
+  }
+  RM_CUDA(h, cudaMemcpyAsync(h->stQ, hostQ, tbytes, cudaMemcpyHostToDevice, h->stream));
+  RM_CUDA(h, cudaMemcpyAsync(h->stK[layer], hostK, tbytes, cudaMemcpyHostToDevice, h->stream));
+  RM_CUDA(h, cudaMemcpyAsync(h->stV[layer], hostV, tbytes, cudaMemcpyHostToDevice, h->stream));
+  s = regmem_attend_frame(h, layer, h->stQ, h->stK[layer], h->stV[layer], h->stOut, h->stSal);
+  if (s != REGMEM_OK) return s;
+  RM_CUDA(h, cudaMemcpyAsync(hostOut, h->stOut, tbytes, cudaMemcpyDeviceToHost, h->stream));
+  RM_CUDA(h, cudaMemcpyAsync(hostSaliency, h->stSal, sbytes, cudaMemcpyDeviceToHost, h->stream));
+  return REGMEM_OK;
+}
+
+regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if (!h->pending[layer])
+    return fail(h, REGMEM_ERR_STATE, "layer %d has no attend pending", layer);
+  if (idx_out && ((reinterpret_cast<uintptr_t>(idx_out) & 3u) != 0))
+    return fail(h, REGMEM_ERR_ARG, "idx_out must be 4-byte aligned");
+  auto* bk = h->bankK + (size_t)layer * h->heads * h->cap * kHeadDim;
+  auto* bv = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
+  if (h->len[layer] == 0) {  // Eq. 4: the first frame is kept whole
+    RM_CUDA(h, launch_anchor(h->pK[layer], h->pV[layer], bk, bv, h->cap, h->N, h->heads, h->stream));
+    h->len[layer] = h->N;
+    h->pending[layer] = 0;
+    return REGMEM_OK;
+  }
+  const int nc = h->N - h->cand_lo;
+  const int kmax = h->budget < nc ? h->budget : nc;
+  if (k < 0 || k > kmax)
+    return fail(h, REGMEM_ERR_ARG, "k = %d outside [0, %d] (budget %d, candidates %d)", k, kmax,
+                h->budget, nc);
+  if (h->len[layer] + k > h->cap)
+    return fail(h, REGMEM_ERR_CAPACITY, "layer %d: %lld + %d rows exceed capacity %lld", layer,
+                h->len[layer], k, h->cap);
+  if (k > 0) {
+    AdmitArgs a;
+    a.sal = h->pS[layer];
+    a.K = h->pK[layer];
+    a.V = h->pV[layer];
+    a.bankK = bk;
+    a.bankV = bv;
+    a.cap = h->cap;
+    a.M = h->len[layer];
+    a.N = h->N;
+    a.H = h->heads;
+    a.cand_lo = h->cand_lo;
+    a.k = k;
+    a.idx_out = idx_out;
+    RM_CUDA(h, launch_admit(a, h->stream));
+  }
+  h->len[layer] += k;
+  h->pending[layer] = 0;
+  return REGMEM_OK;
+}
+
+regmem_status regmem_frame_attention(regmem_t* h, const void* Q, const void* K, const void* V,
+                                     void* out) {
+  regmem_status s = ready(h, 0, false);
+  if (s != REGMEM_OK) return s;
+  if (!Q || !K || !V || !out) return fail(h, REGMEM_ERR_ARG, "null tensor pointer");
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(out))
+    return fail(h, REGMEM_ERR_ARG, "tensor pointers must be 16-byte aligned");
+  return run_attention(h, 0, Q, K, V, out, 0);
+}
+
+regmem_status regmem_reset(regmem_t* h) {
+  if (!h) return REGMEM_ERR_ARG;
+  for (int l = 0; l < h->layers; ++l) {
+    h->len[l] = 0;
+    h->pending[l] = 0;
+  }
+  return REGMEM_OK;
+}
+
+regmem_status regmem_memory_len(const regmem_t* h, int32_t layer, int64_t* len) {
+  if (!h || !len || layer < 0 || layer >= h->layers) return REGMEM_ERR_ARG;
+  *len = h->len[layer];
+  return REGMEM_OK;
+}
+
+regmem_status regmem_capacity(const regmem_t* h, int64_t* rows) {
+  if (!h || !rows) return REGMEM_ERR_ARG;
+  if (!h->frame_set) return REGMEM_ERR_STATE;
+  *rows = h->cap;
+  return REGMEM_OK;
+}
+
+regmem_status regmem_export_bank(regmem_t* h, int32_t layer, void* hostK, void* hostV) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if (!hostK || !hostV) return fail(h, REGMEM_ERR_ARG, "null host pointer");
+  const long long n = h->len[layer];
+  if (n == 0) return REGMEM_OK;
+  const size_t row = kHeadDim * 2;
+  const size_t off = (size_t)layer * h->heads * h->cap * kHeadDim;
+  RM_CUDA(h, cudaMemcpy2DAsync(hostK, n * row, h->bankK + off, h->cap * row, n * row, h->heads,
+                               cudaMemcpyDeviceToHost, h->stream));
+  RM_CUDA(h, cudaMemcpy2DAsync(hostV, n * row, h->bankV + off, h->cap * row, n * row, h->heads,
+                               cudaMemcpyDeviceToHost, h->stream));
+  RM_CUDA(h, cudaStreamSynchronize(h->stream));
+  return check_device_status(h);
+}
+
+regmem_status regmem_import_bank(regmem_t* h, int32_t layer, const void* hostK, const void* hostV,
+                                 int64_t len) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if (len < 0 || len > h->cap)
+    return fail(h, REGMEM_ERR_CAPACITY, "len %lld outside [0, %lld]", (long long)len, h->cap);
+  if (len > 0 && (!hostK || !hostV)) return fail(h, REGMEM_ERR_ARG, "null host pointer");
+  const size_t row = kHeadDim * 2;
+  const size_t off = (size_t)layer * h->heads * h->cap * kHeadDim;
+  if (len > 0) {
+    RM_CUDA(h, cudaMemcpy2DAsync(h->bankK + off, h->cap * row, hostK, len * row, len * row,
+                                 h->heads, cudaMemcpyHostToDevice, h->stream));
+    RM_CUDA(h, cudaMemcpy2DAsync(h->bankV + off, h->cap * row, hostV, len * row, len * row,
+                                 h->heads, cudaMemcpyHostToDevice, h->stream));
+  }
+  RM_CUDA(h, cudaStreamSynchronize(h->stream));
+  h->len[layer] = len;
+  h->pending[layer] = 0;
+  return REGMEM_OK;
+}
+
+regmem_status regmem_copy_lse(regmem_t* h, float* dst) {
+  regmem_status s = ready(h, 0, false);
+  if (s != REGMEM_OK) return s;
+  if (!dst) return fail(h, REGMEM_ERR_ARG, "null pointer");
+  RM_CUDA(h, cudaMemcpyAsync(dst, h->lse, (size_t)h->heads * h->N * sizeof(float),
+                             cudaMemcpyDeviceToDevice, h->stream));
+  return REGMEM_OK;
+}
+
+regmem_status regmem_synchronize(regmem_t* h) {
+  if (!h) return REGMEM_ERR_ARG;
+  if (h->frame_set) {
+    if (cudaSetDevice(h->device) != cudaSuccess)
+      return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
+    RM_CUDA(h, cudaStreamSynchronize(h->stream));
+    RM_CUDA(h, cudaGetLastError());
+  }
+  return check_device_status(h);
+}
+
+void regmem_destroy(regmem_t* h) {
+  if (!h) return;
+  if (h->frame_set) {
+    cudaSetDevice(h->device);
+    cudaStreamSynchronize(h->stream);
+  }
+  cudaFree(h->bankK);
+  cudaFree(h->bankV);
+  cudaFree(h->lse);
+  cudaFree(h->qidx);
+  cudaFree(h->part_o);
+  cudaFree(h->part_lse);
+  if (h->status_host) cudaFreeHost(h->status_host);
+  cudaFree(h->stQ);
+  cudaFree(h->stOut);
+  cudaFree(h->stSal);
+  for (auto* p : h->stK) cudaFree(p);
+  for (auto* p : h->stV) cudaFree(p);
+  delete h;
+}
+
+}  // extern "C"

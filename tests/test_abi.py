@@ -1,0 +1,71 @@
+"""The C-ABI library builds, loads without a GPU and exports exactly the entry
+points include/regmem.h declares (no compute calls here)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "regmem.h")
+
+
+def declared():
+    src = open(HEADER).read()
+    return sorted(set(re.findall(r"REGMEM_API[^;(]*?\b(regmem_\w+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib_path():
+    from paper_2609_23286_gb300 import build
+    return build.build()
+
+
+def test_header_declares_entry_points():
+    names = declared()
+    for n in ("regmem_create", "regmem_attend_frame", "regmem_admit", "regmem_reset",
+              "regmem_destroy", "regmem_set_frame", "regmem_frame_attention"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib_path):
+    out = subprocess.run(["nm", "-D", "--defined-only", lib_path], capture_output=True,
+                         text=True, check=True).stdout
+    exported = sorted(set(re.findall(r"\bT (regmem_\w+)", out)))
+    assert exported == declared()
+
+
+def test_library_loads_without_gpu_and_binding_covers_header(lib_path):
+    from paper_2609_23286_gb300 import regmem
+    lib = regmem.load(lib_path)
+    for n in declared():
+        assert hasattr(lib, n)
+        assert n in regmem._SIGNATURES
+        assert hasattr(regmem, n), f"binding lacks {n}"
+    assert regmem.status_string(regmem.ERR_CAPACITY) == "REGMEM_ERR_CAPACITY"
+
+
+def test_host_side_validation_without_gpu(lib_path):
+    """Argument checks that need no device: bad create arguments, calls before
+    set_frame, null handles."""
+    from paper_2609_23286_gb300 import regmem
+    lib = regmem.load(lib_path)
+    h = ctypes.c_void_p()
+    assert lib.regmem_create(ctypes.byref(h), 0, 1, 64, 1) == regmem.ERR_ARG
+    assert lib.regmem_create(ctypes.byref(h), 1, 1, 96, 1) == regmem.ERR_UNSUPPORTED
+    assert lib.regmem_create(None, 1, 1, 64, 1) == regmem.ERR_ARG
+    handle = regmem.regmem_create(2, 4, 64, 3)
+    try:
+        assert lib.regmem_attend_frame(handle, 0, 16, 16, 16, 16, 16) == regmem.ERR_STATE
+        assert "set_frame" in regmem.regmem_last_error(handle)
+        assert lib.regmem_admit(handle, 0, 1, None) == regmem.ERR_STATE
+        assert regmem.regmem_memory_len(handle, 1) == 0
+        with pytest.raises(regmem.RegmemError):
+            regmem.regmem_memory_len(handle, 2)
+        fd = regmem.FrameDesc(70, 5, 8, 8, 2, 4, 0.0, 0)      # 70 != 5 + 64
+        assert lib.regmem_set_frame(handle, ctypes.byref(fd)) == regmem.ERR_ARG
+        assert lib.regmem_reset(handle) == 0
+    finally:
+        regmem.regmem_destroy(handle)
+    assert lib.regmem_reset(None) == regmem.ERR_ARG

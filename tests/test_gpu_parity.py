@@ -1,0 +1,265 @@
+"""Parity of the CUDA path (through the C ABI) against the fp64 oracle.
+
+Every test feeds both sides the same seeded bf16 inputs.  The oracle gets the
+exact values the GPU saw (bf16 widened to float64)."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from helpers import (Stream, check_indices, check_lse, check_o, check_saliency, to64)
+from paper_2609_23286_gb300 import regmem
+
+pytestmark = pytest.mark.gpu
+
+
+def run_stream(L, H, ns, gh, gw, k, frames, seed, ds=2, check_every=1):
+    """Free-running stream on GPU and oracle; the oracle adopts the GPU's
+    admitted indices after they pass check_indices, so later frames stay
+    comparable.  Returns the number of frames checked."""
+    st = Stream(L, H, ns, gh, gw, budget=k, max_frames=frames, seed=seed, ds=ds)
+    ref = orc.OracleStream(L, H, 64, ns, gh, gw, ds=ds)
+    try:
+        for t in range(1, frames + 1):
+            for layer in range(L):
+                q, kk_, v = st.inputs(layer, t)
+                out, sal, lse = st.attend(layer, q, kk_, v)
+                idx = st.admit(layer, k)
+                torch.cuda.synchronize()
+                r = ref.attend(layer, to64(q), to64(kk_), to64(v))
+                if t % check_every == 0 or t <= 2:
+                    check_o(out, r["O"], f"t={t} l={layer}")
+                    check_lse(lse, r["LSE"], f"t={t} l={layer}")
+                    check_saliency(sal, r["S"], f"t={t} l={layer}")
+                if ref.memory_len(layer) == 0:
+                    ref.admit(layer, k)
+                else:
+                    gi = idx.cpu().numpy().astype(np.int64)
+                    check_indices(gi, to64(sal), r["S"], ns, k, len(ref.qidx))
+                    ref.admit(layer, k, indices=gi)
+                assert st.rm.memory_len(layer) == ref.memory_len(layer) == st.N + (t - 1) * k
+            if t in (1, 2, frames):
+                for layer in range(L):
+                    bk, bv = st.export(layer)
+                    for h in range(H):
+                        assert np.array_equal(bk[h].double().numpy(), ref.bank_k[layer][h])
+                        assert np.array_equal(bv[h].double().numpy(), ref.bank_v[layer][h])
+        st.rm.synchronize()
+    finally:
+        st.close()
+
+
+def test_tiny_stream_full_oracle():
+    """1 layer, 2 heads, 8x8 patches + 5 specials = 69 tokens, 8 frames, k = 1,
+    seed 0: the whole stream against the free-running oracle."""
+    run_stream(1, 2, 5, 8, 8, 1, 8, seed=0)
+
+
+def test_vggt_layer_first_frames():
+    """16 heads, 37x37 + 5 = 1374 tokens, k = 14, seed 1, first 4 frames: several
+    query tiles with a ragged last tile, bank tiles with ragged ends."""
+    run_stream(1, 16, 5, 37, 37, 14, 4, seed=1)
+
+
+def test_two_layers_nonsquare():
+    """37x28 + 5 = 1041 tokens, k = 11, two layers with independent seeds."""
+    run_stream(2, 16, 5, 37, 28, 11, 3, seed=5)
+
+
+@pytest.mark.parametrize("M", [1, 127, 128, 129, 383, 2760])
+def test_teacher_forced_bank_lengths(M):
+    """Single frame against an imported bank of M rows: bank tiles that are
+    tiny, exactly one tile, one row past a tile, and the 100-frame length."""
+    H, ns, gh, gw = 16, 5, 37, 37
+    N = ns + gh * gw
+    st = Stream(1, H, ns, gh, gw, budget=14, max_frames=400, seed=3)
+    try:
+        g = torch.Generator().manual_seed(M)
+        bk = (torch.randn(H, M, 64, generator=g) * 1.3).to(torch.bfloat16)
+        bv = torch.randn(H, M, 64, generator=g).to(torch.bfloat16)
+        st.rm.import_bank(0, bk, bv, M)
+        q, k, v = st.inputs(0, 7)
+        out, sal, lse = st.attend(0, q, k, v)
+        idx = st.admit(0, 14)
+        torch.cuda.synchronize()
+        ref = orc.attend_frame(to64(q), to64(k), to64(v), [bk[h].double().numpy() for h in range(H)],
+                               [bv[h].double().numpy() for h in range(H)], 1 / 8,
+                               orc.sampled_query_tokens(ns, gh, gw, 2))
+        check_o(out, ref["O"], f"M={M}")
+        check_lse(lse, ref["LSE"], f"M={M}")
+        check_saliency(sal, ref["S"], f"M={M}")
+        check_indices(idx.cpu().numpy(), to64(sal), ref["S"], ns, 14, 361)
+        bk2, bv2 = st.export(0)
+        gi = idx.cpu().numpy()
+        for h in range(H):
+            assert torch.equal(bk2[h, :M], bk[h]) and torch.equal(bv2[h, :M], bv[h])
+            assert torch.equal(bk2[h, M:], k[gi[h], h].cpu())
+            assert torch.equal(bv2[h, M:], v[gi[h], h].cpu())
+    finally:
+        st.close()
+
+
+def test_long_bank_sampled_rows():
+    """Config-4 end size: a bank of 29360 rows per head (2000 frames at k = 14).
+    O is checked on sampled query rows (the oracle computes rows one by one),
+    LSE and saliency on all sampled queries / keys."""
+    H, ns, gh, gw = 16, 5, 37, 37
+    N = ns + gh * gw
+    M = N + 1999 * 14
+    st = Stream(1, H, ns, gh, gw, budget=14, max_frames=2001, seed=4)
+    try:
+        g = torch.Generator().manual_seed(11)
+        bk = (torch.randn(H, M, 64, generator=g) * torch.exp(0.5 * torch.randn(1, M, 1, generator=g))).to(torch.bfloat16)
+        bv = torch.randn(H, M, 64, generator=g).to(torch.bfloat16)
+        st.rm.import_bank(0, bk, bv, M)
+        q, k, v = st.inputs(0, 2000)
+        out, sal, lse = st.attend(0, q, k, v)
+        torch.cuda.synchronize()
+        qi = orc.sampled_query_tokens(ns, gh, gw, 2)
+        rows = sorted(set(list(range(0, N, 97)) + [N - 1, 127, 128, 1279, 1280]))
+        q64, k64, v64 = to64(q), to64(k), to64(v)
+        for h in range(H):
+            kc = np.concatenate([bk[h].double().numpy(), k64[:, h]])
+            vc = np.concatenate([bv[h].double().numpy(), v64[:, h]])
+            o_r, l_r, _, _ = orc.attend_head(q64[rows, h], kc, vc, 1 / 8)
+            check_o(out[rows, h], o_r, f"h={h}")
+            check_lse(lse[h, rows], l_r, f"h={h}")
+            _, l_s, z_s, _ = orc.attend_head(q64[qi, h], kc, vc, 1 / 8)
+            s_r = orc.saliency_lse(z_s, l_s, M, list(range(len(qi))))
+            check_saliency(sal[h], s_r, f"h={h}")
+        st.rm.admit(0, 14)
+        st.rm.synchronize()
+    finally:
+        st.close()
+
+
+def test_frame_attention_matches_sdpa_oracle():
+    """Non-causal intra-frame attention (M = 0, no saliency), 1041 tokens."""
+    H, ns, gh, gw = 16, 5, 37, 28
+    st = Stream(1, H, ns, gh, gw, budget=11, max_frames=2, seed=9)
+    try:
+        q, k, v = st.inputs(0, 1)
+        out = torch.empty_like(q)
+        st.rm.frame_attention(q, k, v, out)
+        torch.cuda.synchronize()
+        ref = orc.attend_frame(to64(q), to64(k), to64(v), [np.zeros((0, 64))] * H,
+                               [np.zeros((0, 64))] * H, 1 / 8, [0])
+        check_o(out, ref["O"], "frame attention")
+        assert st.rm.memory_len(0) == 0
+    finally:
+        st.close()
+
+
+def test_k_zero_and_budget_edges():
+    """k = 0 leaves the bank as it is (Eq. 5 layers); k = budget appends."""
+    st = Stream(1, 4, 5, 8, 8, budget=3, max_frames=5, seed=2)
+    try:
+        for t, kk in ((1, 0), (2, 0), (3, 3), (4, 1)):
+            q, k, v = st.inputs(0, t)
+            st.attend(0, q, k, v)
+            st.admit(0, kk)
+        assert st.rm.memory_len(0) == 69 + 0 + 0 + 3 + 1
+        st.rm.synchronize()
+    finally:
+        st.close()
+
+
+def test_host_buffer_entry_point_matches_device_path():
+    H, ns, gh, gw = 16, 5, 37, 37
+    N = ns + gh * gw
+    a = Stream(1, H, ns, gh, gw, budget=14, max_frames=4, seed=6)
+    b = Stream(1, H, ns, gh, gw, budget=14, max_frames=4, seed=6)
+    try:
+        for t in range(1, 4):
+            q, k, v = a.inputs(0, t)
+            out_d, sal_d, _ = a.attend(0, q, k, v)
+            a.admit(0, 14)
+            hq, hk, hv = q.cpu().pin_memory(), k.cpu().pin_memory(), v.cpu().pin_memory()
+            ho = torch.empty_like(hq).pin_memory()
+            hs = torch.empty(H, N, dtype=torch.float32).pin_memory()
+            b.rm.attend_frame_host(0, hq, hk, hv, ho, hs)
+            b.rm.admit(0, 14)
+            b.rm.synchronize()
+            torch.cuda.synchronize()
+            assert torch.equal(ho, out_d.cpu())
+            assert torch.equal(hs, sal_d.cpu())
+    finally:
+        a.close()
+        b.close()
+
+
+def test_deterministic_repeat():
+    """Same inputs twice -> bit-identical outputs, saliency and indices."""
+    res = []
+    for _ in range(2):
+        st = Stream(1, 16, 5, 37, 37, budget=14, max_frames=3, seed=8)
+        try:
+            outs = []
+            for t in (1, 2):
+                q, k, v = st.inputs(0, t)
+                out, sal, lse = st.attend(0, q, k, v)
+                idx = st.admit(0, 14)
+                torch.cuda.synchronize()
+                outs += [out.cpu(), sal.cpu(), idx.cpu()]
+            res.append(outs)
+        finally:
+            st.close()
+    for x, y in zip(*res):
+        assert torch.equal(x, y)
+
+
+def test_state_machine_and_argument_errors():
+    rm = regmem.RegMem(2, 2, 64, 1)
+    try:
+        with pytest.raises(regmem.RegmemError) as e:
+            rm.admit(0, 1)
+        assert e.value.status == regmem.ERR_STATE            # before set_frame
+        rm.set_frame(5, 8, 8, ds=2, max_frames=3)
+        with pytest.raises(regmem.RegmemError) as e:
+            rm.set_frame(5, 8, 8)
+        assert e.value.status == regmem.ERR_STATE            # twice
+        N = 69
+        q = torch.zeros(N, 2, 64, dtype=torch.bfloat16, device="cuda")
+        out = torch.empty_like(q)
+        sal = torch.empty(2, N, device="cuda")
+        with pytest.raises(regmem.RegmemError) as e:
+            rm.admit(0, 1)
+        assert e.value.status == regmem.ERR_STATE            # admit before attend
+        with pytest.raises(regmem.RegmemError) as e:
+            rm.attend_frame(2, q, q, q, out, sal)
+        assert e.value.status == regmem.ERR_ARG              # layer out of range
+        with pytest.raises(regmem.RegmemError) as e:
+            rm.attend_frame(0, q, q, q, None, sal)
+        assert e.value.status == regmem.ERR_ARG              # null pointer
+        with pytest.raises(regmem.RegmemError) as e:
+            rm.attend_frame(0, q.data_ptr() + 2, q, q, out, sal)
+        assert e.value.status == regmem.ERR_ARG              # misaligned
+        rm.attend_frame(0, q, q, q, out, sal)
+        with pytest.raises(regmem.RegmemError) as e:
+            rm.attend_frame(0, q, q, q, out, sal)
+        assert e.value.status == regmem.ERR_STATE            # second attend
+        rm.admit(0, 1)                                       # anchor: k ignored
+        assert rm.memory_len(0) == N
+        for kk in (1, 1):
+            rm.attend_frame(0, q, q, q, out, sal)
+            with pytest.raises(regmem.RegmemError) as e:
+                rm.admit(0, 2)
+            assert e.value.status == regmem.ERR_ARG          # k > budget
+            rm.admit(0, kk)
+        assert rm.memory_len(0) == N + 2 == rm.capacity()
+        rm.attend_frame(0, q, q, q, out, sal)
+        with pytest.raises(regmem.RegmemError) as e:
+            rm.admit(0, 1)
+        assert e.value.status == regmem.ERR_CAPACITY         # bank full
+        assert rm.memory_len(0) == N + 2
+        rm.admit(0, 0)
+        rm.reset()
+        assert rm.memory_len(0) == 0
+        rm.synchronize()
+    finally:
+        rm.close()
+    with pytest.raises(regmem.RegmemError) as e:
+        regmem.regmem_create(1, 1, 128, 1)
+    assert e.value.status == regmem.ERR_UNSUPPORTED
