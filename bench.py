@@ -1,0 +1,507 @@
+#!/usr/bin/env python3
+"""Benchmark of the regulated streaming-attention hot path on GB300.
+
+A step is one frame through every global-attention layer: per layer, the
+regulated attention over [memory ; frame] with LSE (Eq. 3), the LSE-saliency
+(Sec. 3.3) and the top-k admission into the layer's bank (Eq. 4 / Eq. 6).
+Default workload: the long-horizon stream -- 24 layers, 16 heads x 64,
+1374 tokens per frame (37x37 patches + 5 special tokens), k = 14 admitted
+rows per head per frame, 2000 frames, so each layer's memory grows from 0 to
+29,360 rows.  `value` is frames/s over the timed frames (frames 1..K of a
+fresh stream, after W warm-up frames on the same handle followed by a reset).
+
+Inputs: Q/K/V come from a pool of distinct seeded synthetic frames resident
+in HBM (frame t uses pool entry (t-1) mod P); every step touches more than
+L2 holds (>= 202 MB of inputs per frame, plus the banks), so no L2 flush is
+needed.
+
+Also reported:
+  roofline      attention kernel: algorithmic FLOPs / CUDA-event time of its
+                launches in the timed region, against the measured bf16 peak
+  e2e           same metric through regmem_attend_frame_host: pinned host
+                Q/K/V in, O and saliency back to host, copies inside the timed
+                region
+  cpu_baseline  the fp64 oracle on the host cores, timed on a bounded sample
+                (single layer-frames), extrapolated to the stream
+  clocks        nvidia-smi samples taken during the timed region
+
+--impl reference runs only the oracle (the reference arm) on the same
+workload definition.
+Under torchrun with --gpus N each rank runs an independent replica stream
+(distinct seed): weak scaling, no collective on the data path.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "frames/s of regulated attn+saliency+admit at 1374 tok/frame; TC util %"
+UNIT = "frames/s"
+
+CONFIGS = {
+    # name: layers, heads, n_special, grid_h, grid_w, frames, k, seed, frame_attention
+    "tiny": dict(layers=1, heads=2, ns=5, gh=8, gw=8, frames=8, k=1, seed=0, fa=False),
+    "layer": dict(layers=1, heads=16, ns=5, gh=37, gw=37, frames=100, k=14, seed=1, fa=False),
+    "full": dict(layers=24, heads=16, ns=5, gh=37, gw=37, frames=500, k=14, seed=2, fa=False),
+    "long": dict(layers=24, heads=16, ns=5, gh=37, gw=37, frames=2000, k=14, seed=3, fa=False),
+    "nonsquare": dict(layers=24, heads=16, ns=5, gh=37, gw=28, frames=1000, k=11, seed=4, fa=True),
+}
+
+# dram__bytes_read.sum + dram__bytes_write.sum of one attention-kernel launch,
+# from an ncu capture, scaled to the bench workload's mean launch; None until
+# a capture of the current kernel exists.
+ATTN_TRAFFIC_BYTES_PER_LAUNCH = None
+
+
+def describe(cfg, name):
+    N = cfg["ns"] + cfg["gh"] * cfg["gw"]
+    s = (f"{name}: {cfg['layers']} layers x {cfg['heads']} heads x 64, {N} tok/frame "
+         f"({cfg['gh']}x{cfg['gw']} patches + {cfg['ns']} special), k={cfg['k']}/head/frame, "
+         f"{cfg['frames']}-frame stream, 2x2 query sampling")
+    if cfg["fa"]:
+        s += ", each global layer paired with a non-causal frame-attention layer"
+    return s
+
+
+def attended_rows(cfg, t):
+    """L = M + N attended by frame t (memory rows before frame t plus N)."""
+    N = cfg["ns"] + cfg["gh"] * cfg["gw"]
+    M = 0 if t == 1 else N + (t - 2) * cfg["k"]
+    return M + N
+
+
+# ---------------------------------------------------------------------------
+# clocks
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    """nvidia-smi sampling of SM clock, power and throttle reasons."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+
+    def summary(self):
+        return parse_clock_lines(self.lines)
+
+
+def parse_clock_lines(lines):
+    sm, mx, pw, reasons = [], [], [], set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for ln in lines:
+        parts = [p.strip() for p in ln.split(",")]
+        if len(parts) < 7:
+            continue
+        try:
+            sm.append(float(parts[0]))
+            mx.append(float(parts[1]))
+            pw.append(float(parts[2]))
+        except ValueError:
+            continue
+        for n, v in zip(names, parts[3:7]):
+            if v.lower().startswith("active"):
+                reasons.add(n)
+    if not sm:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+    busy = [s for s in sm if s > 0.5 * max(sm)] or sm
+    return {"sm_mhz": statistics.median(busy), "sm_max_mhz": max(mx),
+            "power_w_max": max(pw), "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# distributed helpers (torchrun)
+# ---------------------------------------------------------------------------
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("LOCAL_RANK", "0")), ws
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x: float, device=None) -> float:
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# oracle timing (runs in a fresh process: no CUDA, BLAS threads pinned)
+# ---------------------------------------------------------------------------
+def oracle_layer_frame_seconds(cfg, t, heads=None, seed=7):
+    """Times the fp64 oracle on one layer-frame of the workload at frame t
+    (memory of the size frame t sees, random bf16-valued rows): attention,
+    saliency and top-k for `heads` heads (default all)."""
+    import numpy as np
+    import oracle as orc
+    H = cfg["heads"] if heads is None else heads
+    N = cfg["ns"] + cfg["gh"] * cfg["gw"]
+    M = attended_rows(cfg, t) - N
+    rng = np.random.default_rng(seed + t)
+
+    def bf(a):  # round to bf16-representable values
+        a = a.astype(np.float32)
+        b = (a.view(np.uint32) + 0x7FFF + ((a.view(np.uint32) >> 16) & 1)) & 0xFFFF0000
+        return b.view(np.float32).astype(np.float64)
+
+    q = bf(rng.standard_normal((N, H, 64)))
+    k = bf(rng.standard_normal((N, H, 64)))
+    v = bf(rng.standard_normal((N, H, 64)))
+    bk = [bf(rng.standard_normal((M, 64))) for _ in range(H)]
+    bv = [bf(rng.standard_normal((M, 64))) for _ in range(H)]
+    qidx = orc.sampled_query_tokens(cfg["ns"], cfg["gh"], cfg["gw"], 2)
+    t0 = time.perf_counter()
+    res = orc.attend_frame(q, k, v, bk, bv, 0.125, qidx)
+    for h in range(H):
+        orc.topk_admission(res["S"][h], cfg["ns"], cfg["k"])
+    return time.perf_counter() - t0
+
+
+def oracle_baseline(cfg):
+    """Bounded CPU baseline: single layer-frames at a few stream positions,
+    cost fitted linear in the attended length L and summed over the stream."""
+    frames = cfg["frames"]
+    ts = sorted(set([2, max(2, frames // 2 + 1), frames]))
+    pts = [(attended_rows(cfg, t), oracle_layer_frame_seconds(cfg, t)) for t in ts]
+    if len(pts) >= 2:
+        (l0, s0), (l1, s1) = pts[0], pts[-1]
+        a = (s1 - s0) / (l1 - l0) if l1 != l0 else 0.0
+        b = s0 - a * l0
+    else:
+        a, b = pts[0][1] / pts[0][0], 0.0
+    total = sum(max(a * attended_rows(cfg, t) + b, 0.0) for t in range(1, frames + 1))
+    total *= cfg["layers"] * (2 if cfg["fa"] else 1)
+    return {"frames_per_s": frames / total, "samples": pts}
+
+
+def run_oracle_subprocess(cfg_name, what="baseline", steps=0, warmup=0):
+    threads = os.cpu_count() or 1
+    env = dict(os.environ, OPENBLAS_NUM_THREADS=str(threads), OMP_NUM_THREADS=str(threads),
+               MKL_NUM_THREADS=str(threads), CUDA_VISIBLE_DEVICES="")
+    code = (f"import json, bench; print(json.dumps(bench._oracle_entry({cfg_name!r}, {what!r}, "
+            f"{steps}, {warmup})))")
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True,
+                       text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"oracle timing failed:\n{r.stderr[-2000:]}")
+    out = json.loads(r.stdout.strip().splitlines()[-1])
+    out["threads"] = threads
+    return out
+
+
+def _oracle_entry(cfg_name, what, steps, warmup):
+    cfg = CONFIGS[cfg_name]
+    if what == "baseline":
+        return oracle_baseline(cfg)
+    # reference arm: each step = one (layer, head) of a layer-frame at the
+    # stream's middle frame (mean attended length)
+    t_mid = cfg["frames"] // 2 + 1
+    for _ in range(warmup):
+        oracle_layer_frame_seconds(cfg, t_mid, heads=1)
+    times = [oracle_layer_frame_seconds(cfg, t_mid, heads=1, seed=11 + i) for i in range(steps)]
+    return {"step_s": times, "t_mid": t_mid}
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def make_pool(cfg, P, seed, device):
+    import torch
+    from paper_2609_23286_gb300 import synth
+    N = cfg["ns"] + cfg["gh"] * cfg["gw"]
+    pool = []
+    for layer in range(cfg["layers"]):
+        ks = synth.key_scale(seed, layer, N, device=device)
+        frames = []
+        for f in range(P):
+            frames.append(synth.frame_qkv(seed, layer, f + 1, N, cfg["heads"], 64,
+                                          device=device, scale_cache=ks))
+        pool.append(frames)
+    torch.cuda.synchronize()
+    return pool
+
+
+def run_frames(rm, cfg, pool, t0, count, out, sal, fa_out=None):
+    """Enqueue frames t0 .. t0+count-1 (all layers) through the C ABI."""
+    P = len(pool[0])
+    for t in range(t0, t0 + count):
+        for layer in range(cfg["layers"]):
+            q, k, v = pool[layer][(t - 1) % P]
+            if fa_out is not None:
+                fq, fk, fv = pool[layer][t % P]
+                rm.frame_attention(fq, fk, fv, fa_out)
+            rm.attend_frame(layer, q, k, v, out, sal)
+            rm.admit(layer, cfg["k"])
+
+
+def gpu_arm(args, cfg, cfg_name):
+    import torch
+    import torch.distributed as dist
+    from paper_2609_23286_gb300 import regmem
+
+    rank, local_rank, world = dist_env()
+    if world > 1 and not dist.is_initialized():
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    stream = torch.cuda.current_stream()
+    N = cfg["ns"] + cfg["gh"] * cfg["gw"]
+    H, L = cfg["heads"], cfg["layers"]
+    K = args.steps if args.steps else cfg["frames"]
+    W = args.warmup
+    seed = cfg["seed"] + 1000 * rank
+
+    # CPU baseline first (fresh process, before this process's GPU work grows)
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = run_oracle_subprocess(cfg_name, "baseline")
+
+    P = min(args.pool, max(K, W, 1))
+    pool = make_pool(cfg, P, seed, dev)
+    out = torch.empty(N, H, 64, dtype=torch.bfloat16, device=dev)
+    fa_out = torch.empty_like(out) if cfg["fa"] else None
+    sal = torch.empty(H, N, dtype=torch.float32, device=dev)
+
+    rm = regmem.RegMem(L, H, 64, cfg["k"])
+    rm.set_frame(cfg["ns"], cfg["gh"], cfg["gw"], ds=2, max_frames=max(K, W, 1))
+    rm.set_stream(stream)
+
+    # warm-up frames, then a fresh stream
+    run_frames(rm, cfg, pool, 1, W, out, sal, fa_out)
+    rm.synchronize()
+    rm.reset()
+
+    clocks = ClockSampler(local_rank)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    rm.profile_enable(1)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ev0.record(stream)
+    run_frames(rm, cfg, pool, 1, K, out, sal, fa_out)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clocks.stop()
+    prof = rm.profile_read()
+    ms_local = ev0.elapsed_time(ev1)
+    ms = max_over_ranks(ms_local, dev)
+    mem_rows = rm.memory_len(0)
+
+    # e2e: host buffers through the public host-buffer entry point
+    e2e = None
+    if not args.no_e2e:
+        Ph = min(4, P)
+        hpool = [[tuple(x.cpu().pin_memory() for x in pool[l][f]) for f in range(Ph)]
+                 for l in range(L)]
+        hout = torch.empty(N, H, 64, dtype=torch.bfloat16).pin_memory()
+        hsal = torch.empty(H, N, dtype=torch.float32).pin_memory()
+        hfa = torch.empty_like(hout).pin_memory() if cfg["fa"] else None
+        rm.reset()
+        rm.profile_enable(0)
+        barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for t in range(1, K + 1):
+            for layer in range(L):
+                q, k, v = hpool[layer][(t - 1) % Ph]
+                if hfa is not None:
+                    fq, fk, fv = pool[layer][t % P]
+                    rm.frame_attention(fq, fk, fv, fa_out)  # frame-attention layer: device inputs
+                rm.attend_frame_host(layer, q, k, v, hout, hsal)
+                rm.admit(layer, cfg["k"])
+        e1.record(stream)
+        rm.synchronize()
+        barrier()
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), dev)
+        tb = N * H * 64 * 2
+        e2e = {"value": round(K * world / (e2e_ms / 1e3), 3), "unit": UNIT,
+               "h2d_bytes_per_step": 3 * tb * L, "d2h_bytes_per_step": (tb + H * N * 4) * L,
+               "api": "regmem_attend_frame_host + regmem_admit (pinned host buffers)"}
+
+    launches = int(sum_over_ranks(prof.launches(), dev))
+    rm.close()
+    if rank != 0:
+        return None
+
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except OSError:
+        pass
+    peak_sust = peaks.get("bf16_tflops_sustained")
+    peak_burst = peaks.get("bf16_tflops")
+    peak_src = "measured (MEASURED_PEAKS.json bf16_tflops_sustained: kernel timed inside a long step)"
+    if peak_sust is None:
+        peak_sust, peak_burst, peak_src = 1700.0, 1900.0, "fallback"
+    attn_tflops = prof.attention_flops / (prof.attention_ms / 1e3) / 1e12 if prof.attention_ms else 0.0
+    attn_ms_mean = prof.attention_ms / max(prof.attention_timed, 1)
+    flops_total = sum(4.0 * N * attended_rows(cfg, t) * 64 * H for t in range(1, K + 1)) * L
+    if cfg["fa"]:
+        flops_total += 4.0 * N * N * 64 * H * L * K
+    clk = clocks.summary()
+    line = {
+        "metric": METRIC,
+        "value": round(K * world / (ms / 1e3), 3),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": K,
+        "warmup": W,
+        "ms_per_step": round(ms / K, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) Q/K/V, log-normal(0,0.5) per-token key scale, bf16)",
+        "config": {
+            "workload": describe(cfg, cfg_name),
+            "frames_timed": K,
+            "stream_frames": cfg["frames"],
+            "final_memory_rows_per_head": mem_rows,
+            "input_pool_frames": P,
+            "l2": "no flush: inputs larger than L2 (>= 202 MB of Q/K/V per step plus the banks)",
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+        },
+        "tflops_attention_path": round(flops_total / (ms / 1e3) / 1e12 * world, 2),
+        "roofline": {
+            "kernel": "attn_fwd_kernel (tcgen05 attention + LSE)",
+            "bound": "tensor",
+            "achieved": round(attn_tflops, 2),
+            "peak": peak_sust,
+            "unit": "TFLOP/s",
+            "frac": round(attn_tflops / peak_sust, 4) if peak_sust else None,
+            "frac_of_burst_peak": round(attn_tflops / peak_burst, 4) if peak_burst else None,
+            "peak_source": peak_src,
+            "traffic": ATTN_TRAFFIC_BYTES_PER_LAUNCH,
+            "launches": prof.attention_timed,
+            "mean_launch_ms": round(attn_ms_mean, 5),
+            "algorithmic_flops_per_launch": prof.attention_flops / max(prof.attention_timed, 1),
+            "algorithmic_bytes_per_launch": prof.attention_bytes / max(prof.attention_timed, 1),
+            "share_of_step": round(prof.attention_ms / ms_local, 4) if ms_local else None,
+        },
+        "gpu_launches": launches,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if cpu is not None:
+        line["cpu_baseline"] = {
+            "value": round(cpu["frames_per_s"], 6), "unit": UNIT, "cores": cpu["threads"],
+            "kind": "oracle",
+            "sample": ("fp64 numpy oracle on single layer-frames at stream frames "
+                       + ", ".join(f"L={l} ({s:.2f}s)" for l, s in cpu["samples"])
+                       + f"; cost fitted linear in L and summed over {cfg['frames']} frames x "
+                       f"{L} layers; BLAS matmuls on {cpu['threads']} threads, "
+                       "elementwise exp single-threaded"),
+        }
+    return line
+
+
+def reference_arm(args, cfg, cfg_name):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return None
+    K = args.steps if args.steps else 5
+    W = args.warmup
+    r = run_oracle_subprocess(cfg_name, "reference", K, W)
+    step = statistics.mean(r["step_s"])
+    units = cfg["layers"] * cfg["heads"] * (2 if cfg["fa"] else 1)
+    fps = 1.0 / (step * units)
+    return {
+        "impl": "reference",
+        "metric": METRIC, "value": round(fps, 8), "unit": UNIT, "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": round(step * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": describe(cfg, cfg_name)},
+        "cpu_baseline": {"kind": "oracle", "cores": r["threads"], "value": round(fps, 8),
+                         "unit": UNIT,
+                         "sample": (f"each step = one (layer, head) of a layer-frame at frame "
+                                    f"{r['t_mid']} (mean attended length "
+                                    f"{attended_rows(cfg, r['t_mid'])}); frames/s = 1 / "
+                                    f"({units} x mean step time)")},
+        "e2e": {"value": round(fps, 8), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=0, help="frames timed (default: whole stream)")
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", choices=sorted(CONFIGS), default="long")
+    ap.add_argument("--pool", type=int, default=16, help="distinct input frames kept in HBM")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "ours":
+        ap.error("--warmup must be >= 3")
+    cfg = CONFIGS[args.config]
+    if args.impl == "reference":
+        line = reference_arm(args, cfg, args.config)
+    else:
+        line = gpu_arm(args, cfg, args.config)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

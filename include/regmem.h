@@ -164,6 +164,32 @@ REGMEM_API regmem_status regmem_copy_lse(regmem_t* h, float* dst);
  * status (REGMEM_ERR_TIMEOUT) or CUDA error. */
 REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
 
+/* Launch counters and kernel timing, for measurement tools.
+ * Counters cover every kernel this handle launched since the last
+ * regmem_profile_enable.  When time_attention is set, CUDA events are
+ * recorded on the handle's stream immediately before and after each launch
+ * of the attention kernel (one event pair per attend), and attention_ms is
+ * the sum of those event intervals; the other kernels are not bracketed. */
+typedef struct regmem_profile {
+  int64_t launches_attention; /* attention kernel (attend and frame attention)  */
+  int64_t launches_combine;   /* split-piece merge kernel                       */
+  int64_t launches_saliency;  /* LSE-saliency kernel                            */
+  int64_t launches_admit;     /* top-k + append kernel                          */
+  int64_t launches_anchor;    /* first-frame copy kernel                        */
+  int64_t attention_timed;    /* attention launches with an event pair          */
+  double attention_ms;        /* summed event time of those launches            */
+  double attention_flops;     /* algorithmic 4*N*(M+N)*64*H of those launches   */
+  double attention_bytes;     /* algorithmic HBM bytes of those launches:
+                                 Q, O, K/V of the attended rows, LSE           */
+} regmem_profile;
+
+/* Resets the counters; time_attention = 1 also brackets attention launches
+ * with events (time_attention = 0 stops it). */
+REGMEM_API regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention);
+
+/* Waits for the handle's stream and fills *out. */
+REGMEM_API regmem_status regmem_profile_read(regmem_t* h, regmem_profile* out);
+
 /* Human-readable description of the last error on this handle ("" if none). */
 REGMEM_API const char* regmem_last_error(const regmem_t* h);
 

@@ -430,7 +430,8 @@ int attn_ctas_per_sm() {
   return n < 1 ? 1 : n;
 }
 
-cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s) {
+cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s, cudaEvent_t ev_before,
+                             cudaEvent_t ev_after) {
   Params p;
   p.N = a.N;
   p.H = a.H;
@@ -447,9 +448,13 @@ cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s) {
   p.part_lse = a.part_lse;
   p.status = a.status;
   if (a.grid < 1 || (long long)a.grid > p.total) return cudaErrorInvalidValue;
+  cudaError_t e;
+  if (ev_before && (e = cudaEventRecord(ev_before, s)) != cudaSuccess) return e;
   attn_fwd_kernel<<<a.grid, THREADS, SMEM_BYTES, s>>>(*a.tmQ, *a.tmK, *a.tmV, *a.tmBK, *a.tmBV, p);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess || !combine) return e;
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  if (ev_after && (e = cudaEventRecord(ev_after, s)) != cudaSuccess) return e;
+  if (!combine) return cudaSuccess;
   attn_combine_kernel<<<a.H * p.nqt, 128, 0, s>>>(p, a.grid);
   return cudaGetLastError();
 }

@@ -41,7 +41,10 @@ cudaError_t attn_setup();                              // kernel attributes (onc
 int attn_ctas_per_sm();                                // resident CTAs per SM
 // `combine`: some unit's key range is cut between CTAs, so the partials must
 // be merged (decided on the host from the same schedule formula).
-cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s);
+// ev_before / ev_after (may be null) are recorded around the attention
+// kernel alone.
+cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s,
+                             cudaEvent_t ev_before = nullptr, cudaEvent_t ev_after = nullptr);
 
 // LSE-Saliency over the frame's own keys, per (head, 128-key tile).
 struct SalArgs {

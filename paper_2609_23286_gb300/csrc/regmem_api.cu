@@ -52,6 +52,13 @@ struct regmem {
   float* stSal = nullptr;
   std::vector<__nv_bfloat16*> stK, stV;
 
+  // measurement (regmem_profile_*)
+  regmem_profile prof = {};
+  bool time_attention = false;
+  std::vector<cudaEvent_t> ev_ring;  // pairs: [2i] before, [2i+1] after
+  std::vector<int> ev_busy;
+  size_t ev_next = 0;
+
   std::string err;
 };
 
@@ -145,6 +152,20 @@ regmem_status ready(regmem_t* h, int layer, bool need_layer) {
   return REGMEM_OK;
 }
 
+constexpr size_t kEventPairs = 256;
+
+// Adds the elapsed time of event pair i to the profile and frees the slot.
+cudaError_t harvest_pair(regmem_t* h, size_t i) {
+  cudaError_t e = cudaEventSynchronize(h->ev_ring[2 * i + 1]);
+  if (e != cudaSuccess) return e;
+  float ms = 0.f;
+  e = cudaEventElapsedTime(&ms, h->ev_ring[2 * i], h->ev_ring[2 * i + 1]);
+  if (e != cudaSuccess) return e;
+  h->prof.attention_ms += ms;
+  h->ev_busy[i] = 0;
+  return cudaSuccess;
+}
+
 // Is any (head, query tile) unit's key range cut between two CTAs?
 bool any_split(long long units, long long nkv, long long G) {
   const long long T = units * nkv;
@@ -187,7 +208,32 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   const long long T = (long long)h->heads * nqt * nkv;
   const long long G = T < a.grid ? T : a.grid;
   a.grid = (int)G;
-  RM_CUDA(h, launch_attention(a, any_split((long long)h->heads * nqt, nkv, G), h->stream));
+  const bool combine = any_split((long long)h->heads * nqt, nkv, G);
+  cudaEvent_t eb = nullptr, ea = nullptr;
+  if (h->time_attention) {
+    if (h->ev_ring.empty()) {
+      h->ev_ring.resize(2 * kEventPairs);
+      h->ev_busy.assign(kEventPairs, 0);
+      for (auto& e : h->ev_ring) RM_CUDA(h, cudaEventCreate(&e));
+    }
+    const size_t i = h->ev_next;
+    if (h->ev_busy[i]) RM_CUDA(h, harvest_pair(h, i));
+    eb = h->ev_ring[2 * i];
+    ea = h->ev_ring[2 * i + 1];
+    h->ev_busy[i] = 1;
+    h->ev_next = (i + 1) % kEventPairs;
+  }
+  RM_CUDA(h, launch_attention(a, combine, h->stream, eb, ea));
+  const double L = (double)M + h->N;
+  h->prof.launches_attention += 1;
+  h->prof.launches_combine += combine ? 1 : 0;
+  if (h->time_attention) {
+    h->prof.attention_timed += 1;
+    h->prof.attention_flops += 4.0 * h->N * L * kHeadDim * h->heads;
+    h->prof.attention_bytes += (2.0 * h->N * h->heads * kHeadDim * 2)   // Q in, O out
+                               + (2.0 * L * h->heads * kHeadDim * 2)    // K and V rows
+                               + (4.0 * h->heads * h->N);               // LSE
+  }
   return REGMEM_OK;
 }
 
@@ -335,6 +381,7 @@ regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, con
   sa.sal = saliency;
   sa.status = h->status_dev;
   RM_CUDA(h, launch_saliency(sa, h->stream));
+  h->prof.launches_saliency += 1;
   h->pending[layer] = 1;
   h->pK[layer] = static_cast<const __nv_bfloat16*>(K);
   h->pV[layer] = static_cast<const __nv_bfloat16*>(V);
@@ -384,6 +431,7 @@ regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_o
   auto* bv = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
   if (h->len[layer] == 0) {  // Eq. 4: the first frame is kept whole
     RM_CUDA(h, launch_anchor(h->pK[layer], h->pV[layer], bk, bv, h->cap, h->N, h->heads, h->stream));
+    h->prof.launches_anchor += 1;
     h->len[layer] = h->N;
     h->pending[layer] = 0;
     return REGMEM_OK;
@@ -411,6 +459,7 @@ regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_o
     a.k = k;
     a.idx_out = idx_out;
     RM_CUDA(h, launch_admit(a, h->stream));
+    h->prof.launches_admit += 1;
   }
   h->len[layer] += k;
   h->pending[layer] = 0;
@@ -506,6 +555,32 @@ regmem_status regmem_synchronize(regmem_t* h) {
   return check_device_status(h);
 }
 
+regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention) {
+  if (!h) return REGMEM_ERR_ARG;
+  if (h->frame_set) {
+    if (cudaSetDevice(h->device) != cudaSuccess)
+      return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
+    for (size_t i = 0; i < h->ev_busy.size(); ++i)
+      if (h->ev_busy[i]) RM_CUDA(h, harvest_pair(h, i));
+  }
+  h->prof = regmem_profile{};
+  h->time_attention = time_attention != 0;
+  return REGMEM_OK;
+}
+
+regmem_status regmem_profile_read(regmem_t* h, regmem_profile* out) {
+  if (!h || !out) return REGMEM_ERR_ARG;
+  if (h->frame_set) {
+    if (cudaSetDevice(h->device) != cudaSuccess)
+      return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
+    RM_CUDA(h, cudaStreamSynchronize(h->stream));
+    for (size_t i = 0; i < h->ev_busy.size(); ++i)
+      if (h->ev_busy[i]) RM_CUDA(h, harvest_pair(h, i));
+  }
+  *out = h->prof;
+  return check_device_status(h);
+}
+
 void regmem_destroy(regmem_t* h) {
   if (!h) return;
   if (h->frame_set) {
@@ -524,6 +599,7 @@ void regmem_destroy(regmem_t* h) {
   cudaFree(h->stSal);
   for (auto* p : h->stK) cudaFree(p);
   for (auto* p : h->stV) cudaFree(p);
+  for (auto e : h->ev_ring) cudaEventDestroy(e);
   delete h;
 }
 

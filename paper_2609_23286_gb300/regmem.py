@@ -34,6 +34,8 @@ _SIGNATURES = {
     "regmem_import_bank": (ctypes.c_int, [_P, _I32, _P, _P, ctypes.c_int64]),
     "regmem_copy_lse": (ctypes.c_int, [_P, _P]),
     "regmem_synchronize": (ctypes.c_int, [_P]),
+    "regmem_profile_enable": (ctypes.c_int, [_P, _I32]),
+    "regmem_profile_read": (ctypes.c_int, [_P, _P]),
     "regmem_last_error": (ctypes.c_char_p, [_P]),
     "regmem_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "regmem_destroy": (None, [_P]),
@@ -45,6 +47,22 @@ class FrameDesc(ctypes.Structure):
     _fields_ = [("n_tokens", _I32), ("n_special", _I32), ("grid_h", _I32), ("grid_w", _I32),
                 ("ds", _I32), ("max_frames", _I32), ("scale", ctypes.c_float),
                 ("candidates", _I32)]
+
+
+class Profile(ctypes.Structure):
+    """regmem_profile."""
+    _fields_ = [("launches_attention", ctypes.c_int64), ("launches_combine", ctypes.c_int64),
+                ("launches_saliency", ctypes.c_int64), ("launches_admit", ctypes.c_int64),
+                ("launches_anchor", ctypes.c_int64), ("attention_timed", ctypes.c_int64),
+                ("attention_ms", ctypes.c_double), ("attention_flops", ctypes.c_double),
+                ("attention_bytes", ctypes.c_double)]
+
+    def as_dict(self):
+        return {f: getattr(self, f) for f, _ in self._fields_}
+
+    def launches(self):
+        return (self.launches_attention + self.launches_combine + self.launches_saliency
+                + self.launches_admit + self.launches_anchor)
 
 
 class RegmemError(RuntimeError):
@@ -171,6 +189,16 @@ def regmem_synchronize(h):
     return _check(h, load().regmem_synchronize(h))
 
 
+def regmem_profile_enable(h, time_attention=1):
+    return _check(h, load().regmem_profile_enable(h, int(time_attention)))
+
+
+def regmem_profile_read(h) -> Profile:
+    p = Profile()
+    _check(h, load().regmem_profile_read(h, ctypes.byref(p)))
+    return p
+
+
 def regmem_last_error(h) -> str:
     return load().regmem_last_error(h).decode()
 
@@ -230,6 +258,12 @@ class RegMem:
 
     def synchronize(self):
         return regmem_synchronize(self.h)
+
+    def profile_enable(self, time_attention=1):
+        return regmem_profile_enable(self.h, time_attention)
+
+    def profile_read(self) -> Profile:
+        return regmem_profile_read(self.h)
 
     def close(self):
         if self.h:
