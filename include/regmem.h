@@ -164,6 +164,45 @@ REGMEM_API regmem_status regmem_copy_lse(regmem_t* h, float* dst);
  * status (REGMEM_ERR_TIMEOUT) or CUDA error. */
 REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
 
+/* Allocation-free attend step.  The paper has no counterpart: this entry
+ * point exists for callers that cannot allocate device memory when they run
+ * the attention -- code living inside another framework's memory pool or
+ * arena, plugins handed pre-sized buffers, real-time loops in which a
+ * cudaMalloc could stall on the driver.  It computes what
+ * regmem_attend_frame computes (attention over [bank rows ; frame] and the
+ * LSE-saliency of the frame's keys) with the same kernels, but needs no
+ * handle and allocates nothing: no cudaMalloc, no cudaFree, no allocating
+ * library routine.
+ *
+ * Arguments: fd gives the frame geometry (n_tokens, n_special, grid_h,
+ * grid_w, ds, scale; max_frames and candidates are ignored); Q, K, V, out are
+ * device bf16 [N][heads][64]; bankK/bankV are the caller's device bank of one
+ * layer, bf16 [heads][bank_rows][64], of which the first M rows per head are
+ * attended (NULL allowed when M == 0); saliency is device fp32 [heads][N];
+ * status is an optional device int32 into which the kernels OR nonzero bits if
+ * a bounded device-side wait expires (the caller zeroes it and reads it after
+ * synchronising); stream is a cudaStream_t (NULL: legacy default stream).
+ * All pointers 16-byte aligned (status 4-byte aligned).
+ *
+ * Scratch: the kernels' split partials, LSE rows and sampled-query list live
+ * in one file-scope device array of 22.4 MB that every GPU which loads this
+ * library holds until the process exits.  Limits, rejected with
+ * REGMEM_ERR_UNSUPPORTED before anything is enqueued: heads * N <= 262144,
+ * N <= 65536, sampled queries <= 8192, and the attention grid (2 CTAs per SM)
+ * <= 320 CTAs.  Bad arguments give REGMEM_ERR_ARG; there is no handle, so no
+ * error message is kept.
+ * Every call on a device shares that one array and leaves its contents
+ * behind; calls whose work overlaps on the GPU (two streams, or two host
+ * threads) race on it, so serialise them.  The first call on each device,
+ * with that device current, looks up the array's device address and sets
+ * kernel attributes; make that first call before any stream capture. */
+REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_frame_desc* fd, int32_t heads,
+                                                     const void* Q, const void* K, const void* V,
+                                                     const void* bankK, const void* bankV,
+                                                     int64_t bank_rows, int64_t M, void* out,
+                                                     float* saliency, int32_t* status,
+                                                     void* stream);
+
 /* Launch counters and kernel timing, for measurement tools.
  * Counters cover every kernel this handle launched since the last
  * regmem_profile_enable.  When time_attention is set, CUDA events are

@@ -34,6 +34,8 @@ _SIGNATURES = {
     "regmem_import_bank": (ctypes.c_int, [_P, _I32, _P, _P, ctypes.c_int64]),
     "regmem_copy_lse": (ctypes.c_int, [_P, _P]),
     "regmem_synchronize": (ctypes.c_int, [_P]),
+    "regmem_attend_frame_noalloc": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, ctypes.c_int64,
+                                                   ctypes.c_int64, _P, _P, _P, _P]),
     "regmem_profile_enable": (ctypes.c_int, [_P, _I32]),
     "regmem_profile_read": (ctypes.c_int, [_P, _P]),
     "regmem_last_error": (ctypes.c_char_p, [_P]),
@@ -187,6 +189,20 @@ def regmem_copy_lse(h, dst):
 
 def regmem_synchronize(h):
     return _check(h, load().regmem_synchronize(h))
+
+
+def regmem_attend_frame_noalloc(n_special, grid_h, grid_w, heads, Q, K, V, bankK, bankV,
+                                bank_rows, M, out, saliency, status=None, stream=None, ds=2,
+                                scale=0.0):
+    """Handle-free attend step whose scratch is a fixed device array inside
+    the library (no device allocation)."""
+    fd = FrameDesc(n_special + grid_h * grid_w, n_special, grid_h, grid_w, ds, 1, scale, 0)
+    st = load().regmem_attend_frame_noalloc(ctypes.byref(fd), heads, _ptr(Q), _ptr(K), _ptr(V),
+                                            _ptr(bankK), _ptr(bankV), bank_rows, M, _ptr(out),
+                                            _ptr(saliency), _ptr(status), _stream_ptr(stream))
+    if st < 0:
+        raise RegmemError(st, "regmem_attend_frame_noalloc rejected the call")
+    return st
 
 
 def regmem_profile_enable(h, time_attention=1):
