@@ -230,12 +230,12 @@ def oracle_baseline(cfg):
     return {"frames_per_s": frames / total, "samples": pts}
 
 
-def run_oracle_subprocess(cfg_name, what="baseline", steps=0, warmup=0):
+def run_oracle_subprocess(cfg, what="baseline", steps=0, warmup=0):
     threads = os.cpu_count() or 1
     env = dict(os.environ, OPENBLAS_NUM_THREADS=str(threads), OMP_NUM_THREADS=str(threads),
                MKL_NUM_THREADS=str(threads), CUDA_VISIBLE_DEVICES="")
-    code = (f"import json, bench; print(json.dumps(bench._oracle_entry({cfg_name!r}, {what!r}, "
-            f"{steps}, {warmup})))")
+    code = (f"import json, bench; print(json.dumps(bench._oracle_entry({json.dumps(cfg)!r}, "
+            f"{what!r}, {steps}, {warmup})))")
     r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True,
                        text=True)
     if r.returncode != 0:
@@ -245,8 +245,8 @@ def run_oracle_subprocess(cfg_name, what="baseline", steps=0, warmup=0):
     return out
 
 
-def _oracle_entry(cfg_name, what, steps, warmup):
-    cfg = CONFIGS[cfg_name]
+def _oracle_entry(cfg_json, what, steps, warmup):
+    cfg = json.loads(cfg_json)
     if what == "baseline":
         return oracle_baseline(cfg)
     # reference arm: each step = one (layer, head) of a layer-frame at the
@@ -290,6 +290,18 @@ def run_frames(rm, cfg, pool, t0, count, out, sal, fa_out=None):
             rm.admit(layer, cfg["k"])
 
 
+def synthetic_bank(cfg, rows, seed, device):
+    """Random bf16 bank rows standing in for the memory frame `start` would
+    see: K rows with the per-token log-normal key scale, V rows N(0,1)."""
+    import torch
+    g = torch.Generator(device=device).manual_seed(seed)
+    H = cfg["heads"]
+    k = torch.randn(H, rows, 64, generator=g, device=device)
+    k *= torch.exp(0.5 * torch.randn(1, rows, 1, generator=g, device=device))
+    v = torch.randn(H, rows, 64, generator=g, device=device)
+    return k.to(torch.bfloat16).cpu(), v.to(torch.bfloat16).cpu()
+
+
 def gpu_arm(args, cfg, cfg_name):
     import torch
     import torch.distributed as dist
@@ -303,14 +315,15 @@ def gpu_arm(args, cfg, cfg_name):
     stream = torch.cuda.current_stream()
     N = cfg["ns"] + cfg["gh"] * cfg["gw"]
     H, L = cfg["heads"], cfg["layers"]
-    K = args.steps if args.steps else cfg["frames"]
+    S0 = args.start_frame
+    K = args.steps if args.steps else cfg["frames"] - S0 + 1
     W = args.warmup
     seed = cfg["seed"] + 1000 * rank
 
     # CPU baseline first (fresh process, before this process's GPU work grows)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        cpu = run_oracle_subprocess(cfg_name, "baseline")
+        cpu = run_oracle_subprocess(cfg, "baseline")
 
     P = min(args.pool, max(K, W, 1))
     pool = make_pool(cfg, P, seed, dev)
@@ -319,13 +332,27 @@ def gpu_arm(args, cfg, cfg_name):
     sal = torch.empty(H, N, dtype=torch.float32, device=dev)
 
     rm = regmem.RegMem(L, H, 64, cfg["k"])
-    rm.set_frame(cfg["ns"], cfg["gh"], cfg["gw"], ds=2, max_frames=max(K, W, 1))
+    rm.set_frame(cfg["ns"], cfg["gh"], cfg["gw"], ds=2, max_frames=S0 - 1 + max(K, W, 1))
     rm.set_stream(stream)
 
-    # warm-up frames, then a fresh stream
-    run_frames(rm, cfg, pool, 1, W, out, sal, fa_out)
+    # Starting later in the stream: each layer's bank holds the rows frame S0
+    # would see (synthetic rows), restored again after the warm-up.
+    banks = None
+    if S0 > 1:
+        M0 = attended_rows(cfg, S0) - N
+        banks = [synthetic_bank(cfg, M0, seed * 7919 + l, dev) for l in range(L)]
+
+    def restore():
+        rm.reset()
+        if banks is not None:
+            for l, (bk, bv) in enumerate(banks):
+                rm.import_bank(l, bk, bv, bk.shape[1])
+
+    # warm-up frames, then a fresh stream (or the restored late-stream banks)
+    restore()
+    run_frames(rm, cfg, pool, S0, W, out, sal, fa_out)
     rm.synchronize()
-    rm.reset()
+    restore()
 
     clocks = ClockSampler(local_rank)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -334,7 +361,7 @@ def gpu_arm(args, cfg, cfg_name):
     torch.cuda.synchronize()
     clocks.start()
     ev0.record(stream)
-    run_frames(rm, cfg, pool, 1, K, out, sal, fa_out)
+    run_frames(rm, cfg, pool, S0, K, out, sal, fa_out)
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -353,13 +380,13 @@ def gpu_arm(args, cfg, cfg_name):
         hout = torch.empty(N, H, 64, dtype=torch.bfloat16).pin_memory()
         hsal = torch.empty(H, N, dtype=torch.float32).pin_memory()
         hfa = torch.empty_like(hout).pin_memory() if cfg["fa"] else None
-        rm.reset()
+        restore()
         rm.profile_enable(0)
         barrier()
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for t in range(1, K + 1):
+        for t in range(S0, S0 + K):
             for layer in range(L):
                 q, k, v = hpool[layer][(t - 1) % Ph]
                 if hfa is not None:
@@ -394,7 +421,7 @@ def gpu_arm(args, cfg, cfg_name):
         peak_sust, peak_burst, peak_src = 1700.0, 1900.0, "fallback"
     attn_tflops = prof.attention_flops / (prof.attention_ms / 1e3) / 1e12 if prof.attention_ms else 0.0
     attn_ms_mean = prof.attention_ms / max(prof.attention_timed, 1)
-    flops_total = sum(4.0 * N * attended_rows(cfg, t) * 64 * H for t in range(1, K + 1)) * L
+    flops_total = sum(4.0 * N * attended_rows(cfg, t) * 64 * H for t in range(S0, S0 + K)) * L
     if cfg["fa"]:
         flops_total += 4.0 * N * N * 64 * H * L * K
     clk = clocks.summary()
@@ -414,6 +441,7 @@ def gpu_arm(args, cfg, cfg_name):
         "config": {
             "workload": describe(cfg, cfg_name),
             "frames_timed": K,
+            "first_frame": S0,
             "stream_frames": cfg["frames"],
             "final_memory_rows_per_head": mem_rows,
             "input_pool_frames": P,
@@ -432,6 +460,8 @@ def gpu_arm(args, cfg, cfg_name):
             "peak_source": peak_src,
             "traffic": ATTN_TRAFFIC_BYTES_PER_LAUNCH,
             "launches": prof.attention_timed,
+            "ctas": prof.attention_ctas,
+            "ctas_per_sm": prof.attention_ctas_per_sm,
             "mean_launch_ms": round(attn_ms_mean, 5),
             "algorithmic_flops_per_launch": prof.attention_flops / max(prof.attention_timed, 1),
             "algorithmic_bytes_per_launch": prof.attention_bytes / max(prof.attention_timed, 1),
@@ -460,7 +490,7 @@ def reference_arm(args, cfg, cfg_name):
         return None
     K = args.steps if args.steps else 5
     W = args.warmup
-    r = run_oracle_subprocess(cfg_name, "reference", K, W)
+    r = run_oracle_subprocess(cfg, "reference", K, W)
     step = statistics.mean(r["step_s"])
     units = cfg["layers"] * cfg["heads"] * (2 if cfg["fa"] else 1)
     fps = 1.0 / (step * units)
@@ -489,12 +519,19 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", choices=sorted(CONFIGS), default="long")
     ap.add_argument("--pool", type=int, default=16, help="distinct input frames kept in HBM")
+    ap.add_argument("--start-frame", type=int, default=1,
+                    help="first timed frame; banks are pre-filled with the rows it would see")
+    ap.add_argument("--layers", type=int, default=0, help="override the config's layer count")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be >= 3")
-    cfg = CONFIGS[args.config]
+    cfg = dict(CONFIGS[args.config])
+    if args.layers:
+        cfg["layers"] = args.layers
+    if args.start_frame < 1:
+        ap.error("--start-frame must be >= 1")
     if args.impl == "reference":
         line = reference_arm(args, cfg, args.config)
     else:

@@ -220,6 +220,8 @@ typedef struct regmem_profile {
   double attention_flops;     /* algorithmic 4*N*(M+N)*64*H of those launches   */
   double attention_bytes;     /* algorithmic HBM bytes of those launches:
                                  Q, O, K/V of the attended rows, LSE           */
+  int32_t attention_ctas;     /* grid of the most recent attention launch      */
+  int32_t attention_ctas_per_sm; /* resident attention CTAs per SM (occupancy) */
 } regmem_profile;
 
 /* Resets the counters; time_attention = 1 also brackets attention launches

@@ -39,6 +39,7 @@ inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kTile; 
 
 cudaError_t attn_setup();                              // kernel attributes (once)
 int attn_ctas_per_sm();                                // resident CTAs per SM
+int attn_smem_bytes();                                 // dynamic shared memory per CTA
 // `combine`: some unit's key range is cut between CTAs, so the partials must
 // be merged (decided on the host from the same schedule formula).
 // ev_before / ev_after (may be null) are recorded around the attention

@@ -43,6 +43,7 @@ struct regmem {
   float* part_o = nullptr;    // split-KV partials
   float* part_lse = nullptr;
   int attn_grid = 0;
+  int attn_ctas_per_sm = 0;
   int* status_host = nullptr; // mapped pinned word written by kernels
   int* status_dev = nullptr;
 
@@ -224,6 +225,8 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
     h->ev_next = (i + 1) % kEventPairs;
   }
   RM_CUDA(h, launch_attention(a, combine, h->stream, eb, ea));
+  h->prof.attention_ctas = a.grid;
+  h->prof.attention_ctas_per_sm = h->attn_ctas_per_sm;
   const double L = (double)M + h->N;
   h->prof.launches_attention += 1;
   h->prof.launches_combine += combine ? 1 : 0;
@@ -310,7 +313,8 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   if (!encode_fn()) return fail(h, REGMEM_ERR_CUDA, "cuTensorMapEncodeTiled entry point missing");
 
   const size_t bank_elems = (size_t)h->layers * h->heads * cap * kHeadDim;
-  h->attn_grid = sms * attn_ctas_per_sm();
+  h->attn_ctas_per_sm = attn_ctas_per_sm();
+  h->attn_grid = sms * h->attn_ctas_per_sm;
   RM_CUDA(h, cudaMalloc(&h->bankK, bank_elems * 2));
   RM_CUDA(h, cudaMalloc(&h->bankV, bank_elems * 2));
   RM_CUDA(h, cudaMemset(h->bankK, 0, bank_elems * 2));

@@ -57,7 +57,8 @@ class Profile(ctypes.Structure):
                 ("launches_saliency", ctypes.c_int64), ("launches_admit", ctypes.c_int64),
                 ("launches_anchor", ctypes.c_int64), ("attention_timed", ctypes.c_int64),
                 ("attention_ms", ctypes.c_double), ("attention_flops", ctypes.c_double),
-                ("attention_bytes", ctypes.c_double)]
+                ("attention_bytes", ctypes.c_double), ("attention_ctas", ctypes.c_int32),
+                ("attention_ctas_per_sm", ctypes.c_int32)]
 
     def as_dict(self):
         return {f: getattr(self, f) for f, _ in self._fields_}

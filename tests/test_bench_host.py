@@ -1,0 +1,78 @@
+"""Host-side logic of bench.py, on CPU: multi-rank aggregation over gloo
+(world size 2, as torchrun would launch the replicas), the clock-sample
+parser and the workload arithmetic."""
+import os
+import socket
+
+import pytest
+import torch.multiprocessing as mp
+
+import bench
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, q):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        # each replica's timed region and launch count
+        ms = [120.0, 180.0][rank]
+        launches = [96, 100][rank]
+        bench.barrier()
+        q.put((rank, bench.max_over_ranks(ms), bench.sum_over_ranks(launches), bench.dist_env()))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_rank_aggregation_gloo():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for rank, mx, sm, env in res:
+        assert mx == 180.0          # the slowest replica sets the job time
+        assert sm == 196.0          # launches summed over replicas
+        assert env == (rank, rank, 2)
+
+
+def test_single_process_aggregation_is_identity():
+    assert bench.max_over_ranks(3.5) == 3.5
+    assert bench.sum_over_ranks(7) == 7
+
+
+def test_clock_parser():
+    lines = [
+        "1980, 2070, 650.5, Not Active, Not Active, Not Active, Not Active",
+        "2010, 2070, 700.0, Not Active, Not Active, Not Active, Active",
+        "345, 2070, 120.0, Not Active, Not Active, Not Active, Not Active",   # idle sample
+        "garbage",
+    ]
+    c = bench.parse_clock_lines(lines)
+    assert c["sm_mhz"] == pytest.approx(1995.0)
+    assert c["sm_max_mhz"] == 2070.0
+    assert c["reasons"] == ["sw_power_cap"]
+    assert c["samples"] == 3
+    assert bench.parse_clock_lines([])["sm_mhz"] is None
+
+
+def test_attended_rows_follow_the_growth_law():
+    cfg = bench.CONFIGS["long"]
+    N = 1374
+    assert bench.attended_rows(cfg, 1) == N                     # frame 1: no memory
+    assert bench.attended_rows(cfg, 2) == 2 * N                 # anchor stored whole
+    assert bench.attended_rows(cfg, 2000) - N == N + 1998 * 14  # |M_1999| = N + 1998 k
