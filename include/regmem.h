@@ -188,8 +188,8 @@ REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
  * in one file-scope device array of 22.4 MB that every GPU which loads this
  * library holds until the process exits.  Limits, rejected with
  * REGMEM_ERR_UNSUPPORTED before anything is enqueued: heads * N <= 262144,
- * N <= 65536, sampled queries <= 8192, and the attention grid (2 CTAs per SM)
- * <= 320 CTAs.  Bad arguments give REGMEM_ERR_ARG; there is no handle, so no
+ * N <= 65536, sampled queries <= 8192, and the attention grid (one CTA per
+ * SM) <= 160 CTAs.  Bad arguments give REGMEM_ERR_ARG; there is no handle, so no
  * error message is kept.
  * Every call on a device shares that one array and leaves its contents
  * behind; calls whose work overlaps on the GPU (two streams, or two host

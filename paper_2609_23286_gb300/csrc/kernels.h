@@ -27,15 +27,25 @@ struct AttnArgs {
   float scale;
   __nv_bfloat16* out;       // [N][H][64]
   float* lse;               // [H][N]
-  float* part_o;            // [grid][2][128][64] split-piece partial outputs
-  float* part_lse;          // [grid][2][128]
+  float* part_o;            // [grid][2][kUnitRows][64] split-piece partial outputs
+  float* part_lse;          // [grid][2][kUnitRows]
   int* status;
-  int grid;                 // CTAs of the attention kernel (<= H*nqt*nkv)
+  int grid;                 // CTAs of the attention kernel (<= plan.total)
 };
 
+// Work decomposition: a unit is (head, pair of 128-row query tiles); each
+// unit runs over all key tiles of [bank ; frame].
+constexpr int kUnitRows = 2 * kTile;
+struct AttnPlan {
+  long long units, tiles_per_unit, total;
+};
+AttnPlan attn_plan(int N, int H, int M);
+// Is some unit's key range cut between two of `grid` equal CTA ranges?
+bool attn_any_split(const AttnPlan& pl, long long grid);
+
 // Scratch sizes for a given grid.
-inline size_t attn_part_o_floats(int grid) { return (size_t)grid * 2 * kTile * kHeadDim; }
-inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kTile; }
+inline size_t attn_part_o_floats(int grid) { return (size_t)grid * 2 * kUnitRows * kHeadDim; }
+inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kUnitRows; }
 
 cudaError_t attn_setup();                              // kernel attributes (once)
 int attn_ctas_per_sm();                                // resident CTAs per SM

@@ -24,13 +24,13 @@
 namespace regmem_dev {
 namespace {
 
-constexpr int kMaxCtas = 320;               // split partials for up to 2 CTAs x 160 SMs
+constexpr int kMaxCtas = 160;               // split partials for one CTA on each of up to 160 SMs
 constexpr size_t kMaxLse = 262144;          // heads * tokens per frame
 constexpr int kMaxSampled = 8192;           // sampled queries per frame
 
 struct NoAllocScratch {
-  float part_o[(size_t)kMaxCtas * 2 * kTile * kHeadDim];
-  float part_lse[(size_t)kMaxCtas * 2 * kTile];
+  float part_o[(size_t)kMaxCtas * 2 * kUnitRows * kHeadDim];
+  float part_lse[(size_t)kMaxCtas * 2 * kUnitRows];
   float lse[kMaxLse];
   int qidx[kMaxSampled];
   int status;  // device status bits when the caller passes no status word
@@ -141,11 +141,9 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
   }
   NoAllocScratch* sc = setup.scratch;
 
-  const long long nqt = (N + kTile - 1) / kTile;
-  const long long nkv = (M + kTile - 1) / kTile + nqt;
-  const long long T = (long long)heads * nqt * nkv;
+  const AttnPlan pl = attn_plan(N, heads, (int)M);
   long long G = (long long)setup.sms * setup.ctas_per_sm;
-  if (G > T) G = T;
+  if (G > pl.total) G = pl.total;
   if (G > kMaxCtas) return REGMEM_ERR_UNSUPPORTED;  // more CTAs than the partial scratch holds
 
   CUtensorMap tq, tk, tv, tbk, tbv;
@@ -188,19 +186,7 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
   a.status = st;
   a.grid = (int)G;
   // Same split test as the handle path: is any unit's key range cut between CTAs?
-  bool combine = false;
-  {
-    const long long units = (long long)heads * nqt;
-    auto begin = [&](long long b) { return b * T / G; };
-    auto cta_of = [&](long long x) {
-      long long b = x * G / T;
-      while (b + 1 < G && begin(b + 1) <= x) ++b;
-      while (b > 0 && begin(b) > x) --b;
-      return b;
-    };
-    for (long long u = 0; u < units && !combine; ++u)
-      combine = cta_of(u * nkv) != cta_of(u * nkv + nkv - 1);
-  }
+  const bool combine = attn_any_split(pl, G);
   if (launch_attention(a, combine, stream) != cudaSuccess) return REGMEM_ERR_CUDA;
 
   SalArgs sa;

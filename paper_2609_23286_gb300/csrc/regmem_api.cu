@@ -167,21 +167,6 @@ cudaError_t harvest_pair(regmem_t* h, size_t i) {
   return cudaSuccess;
 }
 
-// Is any (head, query tile) unit's key range cut between two CTAs?
-bool any_split(long long units, long long nkv, long long G) {
-  const long long T = units * nkv;
-  auto begin = [&](long long b) { return b * T / G; };
-  auto cta_of = [&](long long x) {
-    long long b = x * G / T;
-    while (b + 1 < G && begin(b + 1) <= x) ++b;
-    while (b > 0 && begin(b) > x) --b;
-    return b;
-  };
-  for (long long u = 0; u < units; ++u)
-    if (cta_of(u * nkv) != cta_of(u * nkv + nkv - 1)) return true;
-  return false;
-}
-
 regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K, const void* V,
                             void* out, int M) {
   CUtensorMap tq, tk, tv;
@@ -203,13 +188,10 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   a.part_o = h->part_o;
   a.part_lse = h->part_lse;
   a.status = h->status_dev;
-  a.grid = h->attn_grid;
-  const long long nqt = (h->N + kTile - 1) / kTile;
-  const long long nkv = (M + kTile - 1) / kTile + nqt;
-  const long long T = (long long)h->heads * nqt * nkv;
-  const long long G = T < a.grid ? T : a.grid;
+  const AttnPlan pl = attn_plan(h->N, h->heads, M);
+  const long long G = pl.total < h->attn_grid ? pl.total : h->attn_grid;
   a.grid = (int)G;
-  const bool combine = any_split((long long)h->heads * nqt, nkv, G);
+  const bool combine = attn_any_split(pl, G);
   cudaEvent_t eb = nullptr, ea = nullptr;
   if (h->time_attention) {
     if (h->ev_ring.empty()) {
