@@ -16,24 +16,32 @@
 // directly); a unit cut between CTAs leaves normalised fp32 partials
 // (O_p, LSE_p) that attn_combine_kernel merges.
 //
-// CTA layout, warp-specialised (10 warps):
-//   warp 0      TMA producer: both Q tiles of a unit, then K and V tiles
-//               through separate 3-stage rings
-//   warp 1      MMA issuer (one lane) and TMEM owner
-//   warps 2..5  softmax warpgroup 0 -> query tile 0 of the unit
-//   warps 6..9  softmax warpgroup 1 -> query tile 1 of the unit
+// CTA layout, warp-specialised (11 warps):
+//   warp 0       TMA producer: both Q tiles of a unit, then K and V tiles
+//                through separate 5-stage rings
+//   warps 1, 2   MMA issuers, one lane each, for query tile 0 and 1 (each
+//                follows only its own warpgroup's hand-offs, so a slower
+//                warpgroup never holds up the other's MMAs); warp 1 owns TMEM
+//   warps 3..6   softmax warpgroup 0 -> query tile 0 of the unit
+//   warps 7..10  softmax warpgroup 1 -> query tile 1 of the unit
 // Each softmax thread owns one query row (its TMEM lane).  Each key tile is
 // loaded once and serves both query tiles.
-// TMEM (512 columns): S0 [0,128), S1 [128,256) fp32 logits; O0 [256,320),
-// O1 [320,384) fp32 accumulators.  Q K^T is an SS-MMA (Q, K K-major in smem);
-// P is written by the softmax threads to shared memory (bf16, 128-byte
-// swizzled, K-major) and P V is an SS-MMA with V MN-major.
+// TMEM (512 columns): S0 [0,128), S1 [128,256) fp32 logits; P0 [256,320),
+// P1 [320,384) bf16 probabilities packed two per column; O0 [384,448),
+// O1 [448,512) fp32 accumulators.  Q K^T is an SS-MMA (Q, K K-major in smem);
+// P V is a TS-MMA (P from TMEM, V MN-major in smem).  Keeping P in TMEM keeps
+// it off shared memory, whose bandwidth the SS-MMA operand reads and the TMA
+// writes already use up.
 // Hand-offs are mbarriers: s_full (MMA -> softmax, per Q K^T), s_free
 // (softmax -> MMA, S consumed), p_ready (softmax -> MMA, P stored and O
 // rescaled), o_done (MMA -> softmax, per P V), K/V full and empty rings and
-// Q full/empty.  The MMA warp issues Q K^T of the next key tile as soon as
-// S is consumed, so the tensor core computes S(t+1) while the softmax of
-// tile t runs, and the two warpgroups interleave on the tensor core.
+// Q full/empty; the empty barriers take one arrival per issuer, and both
+// issuers wait every phase of the full barriers in order.  Each issuer
+// issues Q K^T of the next key tile as soon as S is consumed, so the tensor
+// core computes S(t+1) while the softmax of tile t runs, and the two query
+// tiles interleave on the tensor core.
+// The softmax uses packed fp32x2 FMA/ADD and three-input max, leaving the
+// exp2 (MUFU) as the dominant instruction stream.
 // The softmax keeps a stale running max and only rescales O when the max
 // grows by more than 2^8, so exp values stay <= 256.
 // Every wait is bounded: on expiry a shared abort word stops all roles, the
@@ -49,12 +57,11 @@ namespace {
 
 constexpr int BM = kTile, BN = kTile, HD = kHeadDim;
 constexpr int UROWS = kUnitRows;         // query rows per unit (two tiles)
-constexpr int KSTAGES = 3, VSTAGES = 3;
+constexpr int KSTAGES = 5, VSTAGES = 5;
 constexpr int TILE_BYTES = BM * HD * 2;  // 16 KB bf16 tile
-constexpr int P_BYTES = BM * BN * 2;     // 32 KB: one query tile's P
-constexpr int THREADS = 320;
+constexpr int THREADS = 352;
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t TM_S0 = 0, TM_S1 = 128, TM_O0 = 256, TM_O1 = 320;
+constexpr uint32_t TM_S0 = 0, TM_S1 = 128, TM_P0 = 256, TM_P1 = 320, TM_O0 = 384, TM_O1 = 448;
 constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s: a hung pipeline gives up
 constexpr uint64_t DRAIN_NS = 200000000ull;   // 0.2 s for draining on abort
 constexpr float RESCALE_LOG2 = 8.0f;
@@ -63,7 +70,6 @@ constexpr uint32_t IDESC_PV = idesc_bf16_f32(128, 64, false, true);
 
 struct Smem {
   uint8_t q[2][TILE_BYTES];
-  uint8_t p[2][P_BYTES];           // per query tile: two 64-key swizzled halves
   uint8_t k[KSTAGES][TILE_BYTES];
   uint8_t v[VSTAGES][TILE_BYTES];
   uint64_t q_full, q_empty;
@@ -136,14 +142,14 @@ __global__ void __launch_bounds__(THREADS, 1)
     sm.abort_flag = 0;
     sm.never = 0;
     mbar_init(smem_addr(&sm.q_full), 1);
-    mbar_init(smem_addr(&sm.q_empty), 1);
+    mbar_init(smem_addr(&sm.q_empty), 2);
     for (int s = 0; s < KSTAGES; ++s) {
       mbar_init(smem_addr(&sm.k_full[s]), 1);
-      mbar_init(smem_addr(&sm.k_empty[s]), 1);
+      mbar_init(smem_addr(&sm.k_empty[s]), 2);
     }
     for (int s = 0; s < VSTAGES; ++s) {
       mbar_init(smem_addr(&sm.v_full[s]), 1);
-      mbar_init(smem_addr(&sm.v_empty[s]), 1);
+      mbar_init(smem_addr(&sm.v_empty[s]), 2);
     }
     for (int t = 0; t < 2; ++t) {
       mbar_init(smem_addr(&sm.s_full[t]), 1);
@@ -151,7 +157,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(smem_addr(&sm.p_ready[t]), BM);
       mbar_init(smem_addr(&sm.o_done[t]), 1);
     }
-    mbar_init(smem_addr(&sm.fin_bar), 1);
+    mbar_init(smem_addr(&sm.fin_bar), 2);
     fence_barrier_init();
   }
   if (warp == 1) {
@@ -212,77 +218,74 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_wait(smem_addr(&sm.v_full[i % VSTAGES]), (i / VSTAGES) & 1, never, DRAIN_NS);
       if (piece > 0) mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, never, DRAIN_NS);
     }
-  } else if (warp == 1) {
-    // ================================================================ MMA issuer
+  } else if (warp == 1 || warp == 2) {
+    // ================================================================ MMA issuers
     if (lane == 0) {
-      const uint32_t sq0 = smem_addr(sm.q[0]), sq1 = smem_addr(sm.q[1]);
-      const uint32_t sp0 = smem_addr(sm.p[0]), sp1 = smem_addr(sm.p[1]);
-      int nqk0 = 0, nqk1 = 0, npv0 = 0, npv1 = 0;  // Q K^T / P V issued per query tile
+      const int t = warp - 1;  // query tile served by this issuer
+      const uint32_t sq = smem_addr(sm.q[t]);
+      const uint32_t d_s = tmem + (t ? TM_S1 : TM_S0), d_p = tmem + (t ? TM_P1 : TM_P0);
+      const uint32_t d_o = tmem + (t ? TM_O1 : TM_O0);
+      const uint32_t b_sfull = smem_addr(&sm.s_full[t]), b_sfree = smem_addr(&sm.s_free[t]);
+      const uint32_t b_pready = smem_addr(&sm.p_ready[t]), b_odone = smem_addr(&sm.o_done[t]);
+      int nqk = 0, npv = 0;  // Q K^T / P V issued for this query tile
       int it = 0, piece = 0;
       bool ok = true;
-      // Q K^T of a key tile for query tile t, once S_t has been consumed.
-      auto qk = [&](int t, uint32_t kaddr) -> bool {
-        int& cnt = t ? nqk1 : nqk0;
-        if (cnt > 0 &&
-            !mbar_wait(smem_addr(&sm.s_free[t]), (cnt - 1) & 1, abort_flag, WAIT_NS))
-          return false;
-        tc_fence_after();
-        const uint32_t qa = t ? sq1 : sq0, d = tmem + (t ? TM_S1 : TM_S0);
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          mma_ss(d, sdesc_sw128(qa + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
-        mma_commit(smem_addr(&sm.s_full[t]));
-        ++cnt;
-        return true;
-      };
-      // P V of a key tile for query tile t, once P_t is stored.
-      auto pv = [&](int t, uint32_t vaddr, bool first) -> bool {
-        int& cnt = t ? npv1 : npv0;
-        if (!mbar_wait(smem_addr(&sm.p_ready[t]), cnt & 1, abort_flag, WAIT_NS)) return false;
-        tc_fence_after();
-        const uint32_t pa = t ? sp1 : sp0, d = tmem + (t ? TM_O1 : TM_O0);
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk)
-          mma_ss(d, sdesc_sw128(pa + (kk >> 2) * (P_BYTES / 2) + (kk & 3) * 32),
-                 sdesc_sw128(vaddr + kk * 2048), IDESC_PV, (first && kk == 0) ? 0u : 1u);
-        mma_commit(smem_addr(&sm.o_done[t]));
-        ++cnt;
-        return true;
-      };
       for (long long x = x_begin; x < x_end && ok;) {
         const Piece pc = piece_at(p, x, x_end);
         const int n = pc.j1 - pc.j0;
-        ok = mbar_wait(smem_addr(&sm.q_full), piece & 1, abort_flag, WAIT_NS);
-        // prologue: Q K^T of the piece's first key tile
-        {
-          const int ks = it % KSTAGES;
-          if (ok) ok = mbar_wait(smem_addr(&sm.k_full[ks]), (it / KSTAGES) & 1, abort_flag, WAIT_NS);
-          if (ok) ok = qk(0, smem_addr(sm.k[ks]));
-          if (ok && pc.has1) ok = qk(1, smem_addr(sm.k[ks]));
-          if (ok) {
-            mma_commit(smem_addr(&sm.k_empty[ks]));
-            if (n == 1) mma_commit(smem_addr(&sm.q_empty));
-          }
-        }
-        for (int jj = 0; jj < n && ok; ++jj, ++it) {
-          if (jj + 1 < n) {  // Q K^T of the next key tile
-            const int ks = (it + 1) % KSTAGES;
-            ok = mbar_wait(smem_addr(&sm.k_full[ks]), ((it + 1) / KSTAGES) & 1, abort_flag, WAIT_NS);
-            if (ok) ok = qk(0, smem_addr(sm.k[ks]));
-            if (ok && pc.has1) ok = qk(1, smem_addr(sm.k[ks]));
-            if (!ok) break;
-            mma_commit(smem_addr(&sm.k_empty[ks]));
-            if (jj + 2 == n) mma_commit(smem_addr(&sm.q_empty));
-          }
-          const int vs = it % VSTAGES;
-          ok = mbar_wait(smem_addr(&sm.v_full[vs]), (it / VSTAGES) & 1, abort_flag, WAIT_NS);
-          if (ok) ok = pv(0, smem_addr(sm.v[vs]), jj == 0);
-          if (ok && pc.has1) ok = pv(1, smem_addr(sm.v[vs]), jj == 0);
-          if (!ok) break;
-          mma_commit(smem_addr(&sm.v_empty[vs]));
-        }
         x += n;
         ++piece;
+        // The tile-1 issuer has nothing to compute for a unit without a second
+        // query tile, but it still waits every phase of the shared full
+        // barriers in order (skipping a phase would let a later parity wait
+        // match an older phase) and releases stages by a plain arrival.
+        const bool act = (t == 0) || pc.has1;
+        auto release = [&](uint32_t bar) {
+          if (act) mma_commit(bar);  // arrives once this issuer's MMAs are done
+          else mbar_arrive(bar);
+        };
+        ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, WAIT_NS);
+        const int t0 = it;  // CTA-local index of the piece's first key tile
+        it += n;
+        // Step jj issues Q K^T of tile jj+1 (as soon as S is free) and then
+        // P V of tile jj (once P is stored); step -1 is the prologue.
+        for (int jj = -1; jj < n && ok; ++jj) {
+          if (jj + 1 < n) {
+            const int tq = t0 + jj + 1;
+            const int ks = tq % KSTAGES;
+            ok = mbar_wait(smem_addr(&sm.k_full[ks]), (tq / KSTAGES) & 1, abort_flag, WAIT_NS);
+            if (ok && act && nqk > 0) ok = mbar_wait(b_sfree, (nqk - 1) & 1, abort_flag, WAIT_NS);
+            if (!ok) break;
+            if (act) {
+              tc_fence_after();
+              const uint32_t kaddr = smem_addr(sm.k[ks]);
+#pragma unroll
+              for (int kk = 0; kk < HD / 16; ++kk)
+                mma_ss(d_s, sdesc_sw128(sq + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
+              mma_commit(b_sfull);
+              ++nqk;
+            }
+            release(smem_addr(&sm.k_empty[ks]));
+            if (jj + 2 == n) release(smem_addr(&sm.q_empty));
+          }
+          if (jj < 0) continue;
+          const int tp = t0 + jj;
+          const int vs = tp % VSTAGES;
+          ok = mbar_wait(smem_addr(&sm.v_full[vs]), (tp / VSTAGES) & 1, abort_flag, WAIT_NS);
+          if (ok && act) ok = mbar_wait(b_pready, npv & 1, abort_flag, WAIT_NS);
+          if (!ok) break;
+          if (act) {
+            tc_fence_after();
+            const uint32_t vaddr = smem_addr(sm.v[vs]);
+#pragma unroll
+            for (int kk = 0; kk < BN / 16; ++kk)  // 16 keys = 8 packed columns of P
+              mma_ts(d_o, d_p + kk * 8, sdesc_sw128(vaddr + kk * 2048), IDESC_PV,
+                     (jj == 0 && kk == 0) ? 0u : 1u);
+            mma_commit(b_odone);
+            ++npv;
+          }
+          release(smem_addr(&sm.v_empty[vs]));
+        }
       }
       // all issued MMAs finish before TMEM and shared memory are released
       mma_commit(smem_addr(&sm.fin_bar));
@@ -290,7 +293,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
   } else {
     // ================================================================ softmax
-    const int t = (warp - 2) >> 2;          // query tile of this warpgroup
+    const int t = (warp - 3) >> 2;          // query tile of this warpgroup
     const int quarter = warp & 3;           // TMEM lane quarter of this warp
     const int row = quarter * 32 + lane;    // query row inside the tile
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
@@ -298,8 +301,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t tm_o = tmem + lane_off + (t ? TM_O1 : TM_O0);
     const uint32_t b_sfull = smem_addr(&sm.s_full[t]), b_sfree = smem_addr(&sm.s_free[t]);
     const uint32_t b_pready = smem_addr(&sm.p_ready[t]), b_odone = smem_addr(&sm.o_done[t]);
-    uint8_t* prow0 = sm.p[t] + row * 128;                // keys 0..63 of this row
-    uint8_t* prow1 = sm.p[t] + P_BYTES / 2 + row * 128;  // keys 64..127
+    const uint32_t tm_p = tmem + lane_off + (t ? TM_P1 : TM_P0);
     const float c = p.scale_log2;
     uint32_t s_phase = 0, o_phase = 0;
     bool stop = false;
@@ -329,13 +331,19 @@ __global__ void __launch_bounds__(THREADS, 1)
           for (int i = 0; i < 128; ++i)
             if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
         }
-        float mx8[8];
+        // row max: four independent chains of three-input max
+        float mx4[4];
 #pragma unroll
-        for (int a = 0; a < 8; ++a) mx8[a] = __uint_as_float(sr[a]);
+        for (int a = 0; a < 4; ++a) mx4[a] = __uint_as_float(sr[a]);
 #pragma unroll
-        for (int i = 8; i < 128; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(sr[i]));
-        const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                               fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+        for (int i = 4; i < 124; i += 8) {
+#pragma unroll
+          for (int a = 0; a < 4; ++a)
+            mx4[a] = fmax3(mx4[a], __uint_as_float(sr[i + 2 * a]), __uint_as_float(sr[i + 2 * a + 1]));
+        }
+        mx4[0] = fmax3(mx4[0], __uint_as_float(sr[124]), __uint_as_float(sr[125]));
+        mx4[1] = fmax3(mx4[1], __uint_as_float(sr[126]), __uint_as_float(sr[127]));
+        const float mx = fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3]));
         const float mnew = mx * c;
         float alpha = 1.f;
         const bool need = mnew > m_used + RESCALE_LOG2;
@@ -344,17 +352,26 @@ __global__ void __launch_bounds__(THREADS, 1)
           l *= alpha;
           m_used = mnew;
         }
-        const float neg = -m_used;
+        // p = exp2(z * c - m_used): packed FMA for the argument, MUFU exp2,
+        // packed ADD for the row sum (two pair accumulators), bf16x2 pack.
+        const uint64_t cc = f2_pack(c, c), nn = f2_pack(-m_used, -m_used);
+        uint64_t acc2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
         uint32_t pk[64];
-        float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int i = 0; i < 64; ++i) {
-          const float p0 = ex2(fmaf(__uint_as_float(sr[2 * i]), c, neg));
-          const float p1 = ex2(fmaf(__uint_as_float(sr[2 * i + 1]), c, neg));
-          ls[i & 3] += p0 + p1;
+          float a0, a1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * i]), __uint_as_float(sr[2 * i + 1])), cc, nn),
+                    a0, a1);
+          const float p0 = ex2(a0), p1 = ex2(a1);
+          acc2[i & 1] = f2_add(acc2[i & 1], f2_pack(p0, p1));
           pk[i] = pack_bf16x2(p0, p1);
         }
-        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        {
+          float s0, s1, s2, s3;
+          f2_unpack(acc2[0], s0, s1);
+          f2_unpack(acc2[1], s2, s3);
+          l += (s0 + s1) + (s2 + s3);
+        }
         if (jj > 0) {
           // P V of the previous key tile must be done before P is overwritten
           // and O is rescaled.
@@ -366,15 +383,11 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           tc_fence_after();
         }
-        // P row -> shared memory, 128-byte swizzled (16-byte chunk g of row r
-        // sits at chunk g ^ (r % 8)), keys 0..63 and 64..127 in two halves.
-#pragma unroll
-        for (int g = 0; g < 8; ++g) {
-          const int cc = (g ^ (row & 7)) * 16;
-          *reinterpret_cast<uint4*>(prow0 + cc) =
-              make_uint4(pk[4 * g], pk[4 * g + 1], pk[4 * g + 2], pk[4 * g + 3]);
-          *reinterpret_cast<uint4*>(prow1 + cc) =
-              make_uint4(pk[32 + 4 * g], pk[32 + 4 * g + 1], pk[32 + 4 * g + 2], pk[32 + 4 * g + 3]);
+        {  // P row -> TMEM (the A operand of the P V MMA)
+          uint32_t (&pa)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pk[0]);
+          uint32_t (&pb)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pk[32]);
+          tmem_st32(tm_p, pa);
+          tmem_st32(tm_p + 32, pb);
         }
         if (jj > 0 && __any_sync(0xffffffffu, need)) {  // rare: the max grew by > 2^8
           uint32_t orr[64];
@@ -386,7 +399,6 @@ __global__ void __launch_bounds__(THREADS, 1)
           tmem_st32(tm_o, oa);
           tmem_st32(tm_o + 32, ob);
         }
-        fence_proxy_async_smem();
         tc_fence_before();
         mbar_arrive(b_pready);
       }
