@@ -185,7 +185,7 @@ REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
  * All pointers 16-byte aligned (status 4-byte aligned).
  *
  * Scratch: the kernels' split partials, LSE rows and sampled-query list live
- * in one file-scope device array of 22.4 MB that every GPU which loads this
+ * in one file-scope device array of 11.8 MB that every GPU which loads this
  * library holds until the process exits.  Limits, rejected with
  * REGMEM_ERR_UNSUPPORTED before anything is enqueued: heads * N <= 262144,
  * N <= 65536, sampled queries <= 8192, and the attention grid (one CTA per
@@ -211,7 +211,6 @@ REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_frame_desc* fd
  * the sum of those event intervals; the other kernels are not bracketed. */
 typedef struct regmem_profile {
   int64_t launches_attention; /* attention kernel (attend and frame attention)  */
-  int64_t launches_combine;   /* split-piece merge kernel                       */
   int64_t launches_saliency;  /* LSE-saliency kernel                            */
   int64_t launches_admit;     /* top-k + append kernel                          */
   int64_t launches_anchor;    /* first-frame copy kernel                        */

@@ -13,8 +13,16 @@
 // consecutive 128-row query tiles); the (unit, key tile) space is cut into
 // `grid` contiguous equal ranges, one per CTA (one CTA per SM).  A unit whose
 // key tiles all fall in one CTA is finished there (O in bf16 and LSE written
-// directly); a unit cut between CTAs leaves normalised fp32 partials
-// (O_p, LSE_p) that attn_combine_kernel merges.
+// directly).  For a unit cut between CTAs, the piece holding its first key
+// tile merges (it is the last piece of its CTA's range, processed after the
+// unit's other pieces, which are the first pieces of the following CTAs):
+// each other piece stores its normalised fp32 partial (O_p, LSE_p) and
+// increments a per-(unit, query tile) counter with release semantics; the
+// merging piece waits (bounded) for the count with acquire loads and folds
+// the partials into its own result,
+//     LSE = log sum_p exp(LSE_p),  O = sum_p exp(LSE_p - LSE) O_p,
+// then resets the counter.  CTAs wait on one another, so the kernel is
+// launched cooperatively (all CTAs resident, one per SM).
 //
 // CTA layout, warp-specialised (11 warps):
 //   warp 0       TMA producer: both Q tiles of a unit, then K and V tiles
@@ -91,8 +99,9 @@ struct Params {
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  float* part_o;
-  float* part_lse;
+  float* part_o;    // [grid][256][64]: the first piece of each CTA, when it is a non-merging piece
+  float* part_lse;  // [grid][256]
+  int* counters;    // [units][2], zero between launches
   int* status;
 };
 
@@ -102,6 +111,14 @@ __device__ __forceinline__ long long range_begin(int b, int G, long long T) {
 
 __device__ __forceinline__ int tile_valid(const Params& p, int j) {
   return j < p.nb ? min(BN, p.M - j * BN) : min(BN, p.N - (j - p.nb) * BN);
+}
+
+// CTA whose range contains global tile x.
+__device__ __forceinline__ int cta_of(long long x, int G, long long T) {
+  long long b = x * G / T;
+  while (b + 1 < G && range_begin((int)b + 1, G, T) <= x) ++b;
+  while (b > 0 && range_begin((int)b, G, T) > x) --b;
+  return (int)b;
 }
 
 // One piece of a CTA's range: unit u, key tiles [j0, j1).
@@ -136,7 +153,6 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   const int G = gridDim.x, b = blockIdx.x;
   const long long x_begin = range_begin(b, G, p.total), x_end = range_begin(b + 1, G, p.total);
-  const int u_first = (int)(x_begin / p.nkv);
 
   if (tid == 0) {
     sm.abort_flag = 0;
@@ -431,15 +447,81 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           p.lse[(size_t)pc.h * p.N + q] = lse_val;
         }
-      } else {
-        const int slot = (pc.u == u_first) ? 0 : 1;
-        const size_t pr = ((size_t)b * 2 + slot) * UROWS + t * BM + row;
+      } else if (pc.j0 > 0) {
+        // a later piece of a split unit: hand the partial to the merging piece
+        const size_t pr = (size_t)b * UROWS + t * BM + row;
         float4* dst = reinterpret_cast<float4*>(p.part_o + pr * HD);
 #pragma unroll
         for (int c4 = 0; c4 < 16; ++c4)
           dst[c4] = make_float4(__uint_as_float(orr[c4 * 4 + 0]) * inv_l, __uint_as_float(orr[c4 * 4 + 1]) * inv_l,
                                 __uint_as_float(orr[c4 * 4 + 2]) * inv_l, __uint_as_float(orr[c4 * 4 + 3]) * inv_l);
         p.part_lse[pr] = lse_val;
+        named_bar_sync(1 + t, BM);
+        if ((warp & 3) == 3 && lane == 0) red_release_add(&p.counters[pc.u * 2 + t], 1);
+      } else {
+        // first piece of a split unit: wait for the other pieces and merge
+        const long long T = p.total;
+        const int b_hi = cta_of((long long)pc.u * p.nkv + p.nkv - 1, G, T);
+        const int others = b_hi - b;  // pieces in CTAs b+1 .. b_hi
+        const bool leader = (warp & 3) == 3 && lane == 0;
+        if (leader) {
+          int* cnt = &p.counters[pc.u * 2 + t];
+          bool done = ld_acquire(cnt) >= others;
+          const uint64_t t0 = done ? 0 : globaltimer_ns();
+          while (!done) {
+            if (*abort_flag || globaltimer_ns() - t0 > WAIT_NS) {
+              *abort_flag = 1;
+              break;
+            }
+            __nanosleep(64);
+            done = ld_acquire(cnt) >= others;
+          }
+          *cnt = 0;  // every other piece has counted: ready for the next launch
+        }
+        named_bar_sync(1 + t, BM);
+        if (*abort_flag) {
+          stop = true;
+        } else {
+          // online merge: own result first, then the partials in CTA order
+          float m = lse_val, den = 1.f;
+          float acc[HD];
+#pragma unroll
+          for (int i = 0; i < HD; ++i) acc[i] = __uint_as_float(orr[i]) * inv_l;
+          for (int bb = b + 1; bb <= b_hi; ++bb) {
+            const size_t pr = (size_t)bb * UROWS + t * BM + row;
+            const float lp = __ldcg(p.part_lse + pr);
+            const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD);
+            float4 v[16];
+#pragma unroll
+            for (int c4 = 0; c4 < 16; ++c4) v[c4] = __ldcg(src + c4);
+            const float mn = fmaxf(m, lp);
+            const float a_old = ex2((m - mn) * 1.4426950408889634f);
+            const float a_new = ex2((lp - mn) * 1.4426950408889634f);
+            den = den * a_old + a_new;
+#pragma unroll
+            for (int c4 = 0; c4 < 16; ++c4) {
+              acc[c4 * 4 + 0] = acc[c4 * 4 + 0] * a_old + v[c4].x * a_new;
+              acc[c4 * 4 + 1] = acc[c4 * 4 + 1] * a_old + v[c4].y * a_new;
+              acc[c4 * 4 + 2] = acc[c4 * 4 + 2] * a_old + v[c4].z * a_new;
+              acc[c4 * 4 + 3] = acc[c4 * 4 + 3] * a_old + v[c4].w * a_new;
+            }
+            m = mn;
+          }
+          const float inv = 1.f / den;
+          if (q < p.N) {
+            uint4* o = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + pc.h) * HD);
+#pragma unroll
+            for (int c8 = 0; c8 < 8; ++c8) {
+              uint4 w4;
+              w4.x = pack_bf16x2(acc[c8 * 8 + 0] * inv, acc[c8 * 8 + 1] * inv);
+              w4.y = pack_bf16x2(acc[c8 * 8 + 2] * inv, acc[c8 * 8 + 3] * inv);
+              w4.z = pack_bf16x2(acc[c8 * 8 + 4] * inv, acc[c8 * 8 + 5] * inv);
+              w4.w = pack_bf16x2(acc[c8 * 8 + 6] * inv, acc[c8 * 8 + 7] * inv);
+              o[c8] = w4;
+            }
+            p.lse[(size_t)pc.h * p.N + q] = m + __logf(den);
+          }
+        }
       }
     }
   }
@@ -450,65 +532,6 @@ __global__ void __launch_bounds__(THREADS, 1)
     tmem_dealloc(tmem, TMEM_COLS);
   }
   if (tid == 0 && sm.abort_flag) atomicOr(p.status, kStatusTimeout);
-}
-
-// Merges the partial (O_p, LSE_p) of every unit whose key tiles were split
-// across CTAs:  LSE = log sum_p exp(LSE_p),  O = sum_p exp(LSE_p - LSE) O_p.
-__global__ void __launch_bounds__(UROWS) attn_combine_kernel(Params p, int G) {
-  const int u = blockIdx.x;
-  const long long T = p.total;
-  const int nkv = p.nkv;
-  auto cta_of = [&](long long x) {
-    long long bb = x * G / T;
-    while (bb + 1 < G && range_begin((int)bb + 1, G, T) <= x) ++bb;
-    while (bb > 0 && range_begin((int)bb, G, T) > x) --bb;
-    return (int)bb;
-  };
-  const int b_lo = cta_of((long long)u * nkv), b_hi = cta_of((long long)u * nkv + nkv - 1);
-  if (b_lo == b_hi) return;  // finished inside one CTA
-  const int h = u / p.nqp, qp = u - h * p.nqp;
-  const int r = threadIdx.x;  // row inside the unit
-  const int q = 2 * qp * BM + r;
-  if (q >= p.N) return;
-  float mx = -INFINITY;
-  for (int bb = b_lo; bb <= b_hi; ++bb) {
-    const int slot = (u == (int)(range_begin(bb, G, T) / nkv)) ? 0 : 1;
-    mx = fmaxf(mx, p.part_lse[((size_t)bb * 2 + slot) * UROWS + r]);
-  }
-  float den = 0.f;
-  for (int bb = b_lo; bb <= b_hi; ++bb) {
-    const int slot = (u == (int)(range_begin(bb, G, T) / nkv)) ? 0 : 1;
-    den += __expf(p.part_lse[((size_t)bb * 2 + slot) * UROWS + r] - mx);
-  }
-  const float lse = mx + __logf(den);
-  float acc[HD];
-#pragma unroll
-  for (int i = 0; i < HD; ++i) acc[i] = 0.f;
-  for (int bb = b_lo; bb <= b_hi; ++bb) {
-    const int slot = (u == (int)(range_begin(bb, G, T) / nkv)) ? 0 : 1;
-    const size_t pr = ((size_t)bb * 2 + slot) * UROWS + r;
-    const float w = __expf(p.part_lse[pr] - lse);
-    const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD);
-#pragma unroll
-    for (int c4 = 0; c4 < 16; ++c4) {
-      const float4 v = src[c4];
-      acc[c4 * 4 + 0] += w * v.x;
-      acc[c4 * 4 + 1] += w * v.y;
-      acc[c4 * 4 + 2] += w * v.z;
-      acc[c4 * 4 + 3] += w * v.w;
-    }
-  }
-  uint4* dst = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + h) * HD);
-#pragma unroll
-  for (int c8 = 0; c8 < 8; ++c8) {
-    uint4 w;
-    w.x = pack_bf16x2(acc[c8 * 8 + 0], acc[c8 * 8 + 1]);
-    w.y = pack_bf16x2(acc[c8 * 8 + 2], acc[c8 * 8 + 3]);
-    w.z = pack_bf16x2(acc[c8 * 8 + 4], acc[c8 * 8 + 5]);
-    w.w = pack_bf16x2(acc[c8 * 8 + 6], acc[c8 * 8 + 7]);
-    dst[c8] = w;
-  }
-  p.lse[(size_t)h * p.N + q] = lse;
 }
 
 Params make_params(const AttnArgs& a) {
@@ -527,6 +550,7 @@ Params make_params(const AttnArgs& a) {
   p.lse = a.lse;
   p.part_o = a.part_o;
   p.part_lse = a.part_lse;
+  p.counters = a.counters;
   p.status = a.status;
   return p;
 }
@@ -539,20 +563,6 @@ AttnPlan attn_plan(int N, int H, int M) {
   pl.tiles_per_unit = (M + BN - 1) / BN + (N + BN - 1) / BN;
   pl.total = pl.units * pl.tiles_per_unit;
   return pl;
-}
-
-bool attn_any_split(const AttnPlan& pl, long long G) {
-  const long long T = pl.total, nkv = pl.tiles_per_unit;
-  auto begin = [&](long long b) { return b * T / G; };
-  auto cta_of = [&](long long x) {
-    long long b = x * G / T;
-    while (b + 1 < G && begin(b + 1) <= x) ++b;
-    while (b > 0 && begin(b) > x) --b;
-    return b;
-  };
-  for (long long u = 0; u < pl.units; ++u)
-    if (cta_of(u * nkv) != cta_of(u * nkv + nkv - 1)) return true;
-  return false;
 }
 
 cudaError_t attn_setup() {
@@ -572,19 +582,28 @@ int attn_ctas_per_sm() {
 
 int attn_smem_bytes() { return (int)SMEM_BYTES; }
 
-cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s, cudaEvent_t ev_before,
+cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_before,
                              cudaEvent_t ev_after) {
   const Params p = make_params(a);
   if (a.grid < 1 || (long long)a.grid > p.total) return cudaErrorInvalidValue;
   cudaError_t e;
   if (ev_before && (e = cudaEventRecord(ev_before, s)) != cudaSuccess) return e;
-  attn_fwd_kernel<<<a.grid, THREADS, SMEM_BYTES, s>>>(*a.tmQ, *a.tmK, *a.tmV, *a.tmBK, *a.tmBV, p);
-  e = cudaGetLastError();
+  // Cooperative: the merging pieces wait for pieces of other CTAs, so every
+  // CTA must be resident (the launch fails rather than oversubscribe).
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.grid);
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, attn_fwd_kernel, *a.tmQ, *a.tmK, *a.tmV, *a.tmBK, *a.tmBV, p);
   if (e != cudaSuccess) return e;
   if (ev_after && (e = cudaEventRecord(ev_after, s)) != cudaSuccess) return e;
-  if (!combine) return cudaSuccess;
-  attn_combine_kernel<<<(int)(a.H * (long long)p.nqp), UROWS, 0, s>>>(p, a.grid);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 }  // namespace regmem_dev

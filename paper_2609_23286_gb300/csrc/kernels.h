@@ -27,8 +27,9 @@ struct AttnArgs {
   float scale;
   __nv_bfloat16* out;       // [N][H][64]
   float* lse;               // [H][N]
-  float* part_o;            // [grid][2][kUnitRows][64] split-piece partial outputs
-  float* part_lse;          // [grid][2][kUnitRows]
+  float* part_o;            // [grid][kUnitRows][64] split-piece partial outputs
+  float* part_lse;          // [grid][kUnitRows]
+  int* counters;            // [units][2] piece counters, all zero between launches
   int* status;
   int grid;                 // CTAs of the attention kernel (<= plan.total)
 };
@@ -40,22 +41,17 @@ struct AttnPlan {
   long long units, tiles_per_unit, total;
 };
 AttnPlan attn_plan(int N, int H, int M);
-// Is some unit's key range cut between two of `grid` equal CTA ranges?
-bool attn_any_split(const AttnPlan& pl, long long grid);
 
 // Scratch sizes for a given grid.
-inline size_t attn_part_o_floats(int grid) { return (size_t)grid * 2 * kUnitRows * kHeadDim; }
-inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kUnitRows; }
+inline size_t attn_part_o_floats(int grid) { return (size_t)grid * kUnitRows * kHeadDim; }
+inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * kUnitRows; }
 
 cudaError_t attn_setup();                              // kernel attributes (once)
 int attn_ctas_per_sm();                                // resident CTAs per SM
 int attn_smem_bytes();                                 // dynamic shared memory per CTA
-// `combine`: some unit's key range is cut between CTAs, so the partials must
-// be merged (decided on the host from the same schedule formula).
-// ev_before / ev_after (may be null) are recorded around the attention
-// kernel alone.
-cudaError_t launch_attention(const AttnArgs& a, bool combine, cudaStream_t s,
-                             cudaEvent_t ev_before = nullptr, cudaEvent_t ev_after = nullptr);
+// ev_before / ev_after (may be null) are recorded around the attention kernel.
+cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_before = nullptr,
+                             cudaEvent_t ev_after = nullptr);
 
 // LSE-Saliency over the frame's own keys, per (head, 128-key tile).
 struct SalArgs {

@@ -42,6 +42,7 @@ struct regmem {
   int* qidx = nullptr;        // [nq]
   float* part_o = nullptr;    // split-KV partials
   float* part_lse = nullptr;
+  int* counters = nullptr;    // split-piece counters, [units][2]
   int attn_grid = 0;
   int attn_ctas_per_sm = 0;
   int* status_host = nullptr; // mapped pinned word written by kernels
@@ -187,11 +188,11 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   a.lse = h->lse;
   a.part_o = h->part_o;
   a.part_lse = h->part_lse;
+  a.counters = h->counters;
   a.status = h->status_dev;
   const AttnPlan pl = attn_plan(h->N, h->heads, M);
   const long long G = pl.total < h->attn_grid ? pl.total : h->attn_grid;
   a.grid = (int)G;
-  const bool combine = attn_any_split(pl, G);
   cudaEvent_t eb = nullptr, ea = nullptr;
   if (h->time_attention) {
     if (h->ev_ring.empty()) {
@@ -206,12 +207,11 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
     h->ev_busy[i] = 1;
     h->ev_next = (i + 1) % kEventPairs;
   }
-  RM_CUDA(h, launch_attention(a, combine, h->stream, eb, ea));
+  RM_CUDA(h, launch_attention(a, h->stream, eb, ea));
   h->prof.attention_ctas = a.grid;
   h->prof.attention_ctas_per_sm = h->attn_ctas_per_sm;
   const double L = (double)M + h->N;
   h->prof.launches_attention += 1;
-  h->prof.launches_combine += combine ? 1 : 0;
   if (h->time_attention) {
     h->prof.attention_timed += 1;
     h->prof.attention_flops += 4.0 * h->N * L * kHeadDim * h->heads;
@@ -306,6 +306,9 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
   RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_floats(h->attn_grid) * sizeof(float)));
   RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid) * sizeof(float)));
+  const size_t n_counters = (size_t)attn_plan(N, h->heads, 0).units * 2;
+  RM_CUDA(h, cudaMalloc(&h->counters, n_counters * sizeof(int)));
+  RM_CUDA(h, cudaMemset(h->counters, 0, n_counters * sizeof(int)));
   RM_CUDA(h, cudaHostAlloc(&h->status_host, sizeof(int), cudaHostAllocMapped));
   *h->status_host = 0;
   RM_CUDA(h, cudaHostGetDevicePointer(&h->status_dev, h->status_host, 0));
@@ -579,6 +582,7 @@ void regmem_destroy(regmem_t* h) {
   cudaFree(h->qidx);
   cudaFree(h->part_o);
   cudaFree(h->part_lse);
+  cudaFree(h->counters);
   if (h->status_host) cudaFreeHost(h->status_host);
   cudaFree(h->stQ);
   cudaFree(h->stOut);

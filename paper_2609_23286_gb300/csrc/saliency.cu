@@ -10,9 +10,11 @@
 // the paper becomes a private sum over its row: no cross-thread reduction and
 // a fixed summation order (deterministic).  exp is taken in fp32 on the exact
 // fp32 logits, never on the bf16 P of the attention kernel.
-// The key tile arrives by TMA; sampled query rows are gathered with 16-byte
-// loads into a 128-byte-swizzled tile, two chunks double-buffered so the next
-// chunk's MMA overlaps the current chunk's exponentials.
+// The key tile arrives by TMA while every thread gathers its sampled query
+// rows with 16-byte cp.async copies into 128-byte-swizzled tiles; up to four
+// 128-query chunks are resident at once.  Z^T alternates between two
+// 128-column TMEM buffers: the MMA of chunk c+2 is issued as soon as every
+// thread has read chunk c, so it runs under the exponentials of chunk c.
 
 #include "kernels.h"
 #include "ptx.cuh"
@@ -25,7 +27,8 @@ namespace {
 constexpr int BT = kTile, HD = kHeadDim;
 constexpr int TILE_BYTES = BT * HD * 2;
 constexpr int THREADS = 128;
-constexpr uint32_t TMEM_COLS = 256;  // two 128-column Z^T buffers
+constexpr int QS = 4;                 // resident sampled-query chunks
+constexpr uint32_t TMEM_COLS = 256;   // two 128-column Z^T buffers
 constexpr uint64_t WAIT_NS = 2000000000ull;
 constexpr uint64_t DRAIN_NS = 200000000ull;
 constexpr uint32_t IDESC = idesc_bf16_f32(128, 128, false, false);
@@ -33,16 +36,16 @@ constexpr int MAX_CHUNKS = 64;  // sampled queries <= 8192
 
 struct Smem {
   uint8_t k[TILE_BYTES];
-  uint8_t qs[2][TILE_BYTES];
-  float lse2[2][BT];
+  uint8_t qs[QS][TILE_BYTES];
+  float lse2[QS][BT];
   uint64_t k_full, mma_bar[2], fin_bar;
   uint32_t tmem_base;
   int abort_flag;
   int never;
 };
-// At least 80 KB so no more than two CTAs share an SM: two 256-column TMEM
-// allocations fill the SM's 512 columns.
-constexpr size_t SMEM_BYTES = (sizeof(Smem) + 1024 > 80 * 1024) ? sizeof(Smem) + 1024 : 80 * 1024;
+// About 83 KB: at most two CTAs share an SM, so their two 256-column TMEM
+// allocations fit the SM's 512 columns.
+constexpr size_t SMEM_BYTES = sizeof(Smem) + 1024;
 
 struct Params {
   const __nv_bfloat16* Q;
@@ -55,28 +58,33 @@ struct Params {
   int* status;
 };
 
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
 // Gather sampled query rows [chunk*128, chunk*128+128) of head h into a
-// swizzled K-major tile, and their LSE (in log2 units) into lse2.  Rows past
-// nq are zero with lse2 = +inf, so they contribute exp2(-inf) = 0.
+// swizzled K-major tile (16-byte chunk c of row r at chunk c ^ (r % 8)), and
+// their LSE (log2 units) into lse2.  Rows past nq are zero with lse2 = +inf,
+// so they contribute exp2(-inf) = 0.
 __device__ __forceinline__ void gather_chunk(const Params& p, int h, int chunk, uint8_t* tile,
                                              float* lse2, int tid) {
   const int i = chunk * BT + tid;  // one sampled row per thread
-  uint4 v[8];
-  float l2 = INFINITY;
+  const uint32_t base = smem_addr(tile) + tid * 128;
   if (i < p.nq) {
     const int tok = p.qidx[i];
     const uint4* src = reinterpret_cast<const uint4*>(p.Q + ((size_t)tok * p.H + h) * HD);
 #pragma unroll
-    for (int c = 0; c < 8; ++c) v[c] = src[c];
-    l2 = p.lse[(size_t)h * p.N + tok] * 1.4426950408889634f;
+    for (int c = 0; c < 8; ++c) cp_async16(base + ((c ^ (tid & 7)) * 16), src + c);
+    lse2[tid] = p.lse[(size_t)h * p.N + tok] * 1.4426950408889634f;
   } else {
 #pragma unroll
-    for (int c = 0; c < 8; ++c) v[c] = make_uint4(0, 0, 0, 0);
+    for (int c = 0; c < 8; ++c)
+      *reinterpret_cast<uint4*>(tile + tid * 128 + c * 16) = make_uint4(0, 0, 0, 0);
+    lse2[tid] = INFINITY;
   }
-#pragma unroll
-  for (int c = 0; c < 8; ++c)
-    *reinterpret_cast<uint4*>(tile + tid * 128 + ((c ^ (tid & 7)) * 16)) = v[c];
-  lse2[tid] = l2;
 }
 
 __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant__ CUtensorMap tmK,
@@ -84,7 +92,7 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
   extern __shared__ uint8_t smem_raw[];
   const uintptr_t raw = reinterpret_cast<uintptr_t>(smem_raw);
   Smem& sm = *reinterpret_cast<Smem*>((raw + 1023) & ~uintptr_t(1023));
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tid = threadIdx.x, warp = tid >> 5;
   const int nkt = (p.N + BT - 1) / BT;
   const int h = blockIdx.x / nkt, kt = blockIdx.x - h * nkt;
   const int nchunks = (p.nq + BT - 1) / BT;
@@ -92,8 +100,9 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
   volatile int* never = &sm.never;
   const uint32_t b_k = smem_addr(&sm.k_full), b_fin = smem_addr(&sm.fin_bar);
   const uint32_t b_mma[2] = {smem_addr(&sm.mma_bar[0]), smem_addr(&sm.mma_bar[1])};
+  const bool issuer = (tid == 0);
 
-  if (tid == 0) {
+  if (issuer) {
     sm.abort_flag = 0;
     sm.never = 0;
     mbar_init(b_k, 1);
@@ -108,68 +117,75 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
     tmem_alloc(smem_addr(&sm.tmem_base), TMEM_COLS);
     tmem_relinquish();
   }
-  if (nchunks > 0) gather_chunk(p, h, 0, sm.qs[0], sm.lse2[0], tid);
-  fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   const uint32_t lane_off = (uint32_t)(warp * 32) << 16;
-  const bool elected = (tid == 0);
   bool k_ok = true;
-  if (elected) {
-    k_ok = mbar_wait(b_k, 0, abort_flag, WAIT_NS);
-    if (k_ok && nchunks > 0) {
-#pragma unroll
-      for (int kk = 0; kk < HD / 16; ++kk)
-        mma_ss(tmem, sdesc_sw128(smem_addr(sm.k) + kk * 32), sdesc_sw128(smem_addr(sm.qs[0]) + kk * 32),
-               IDESC, kk > 0);
-    }
-    mma_commit(b_mma[0]);
-  }
   float acc = 0.f;
   uint32_t ph[2] = {0u, 0u};
-  for (int ch = 0; ch < nchunks; ++ch) {
-    const int buf = ch & 1;
-    const bool ok = mbar_wait(b_mma[buf], ph[buf], abort_flag, WAIT_NS);
-    ph[buf] ^= 1;
-    tc_fence_before();
-    // After this barrier every thread is done with chunk ch-1 (its Z^T load
-    // and its lse2 reads) and the MMA of chunk ch-1 has completed, so the
-    // other buffers can be refilled for chunk ch+1.
-    if (__syncthreads_or(!ok || *abort_flag)) break;
-    if (ch + 1 < nchunks) {
-      gather_chunk(p, h, ch + 1, sm.qs[buf ^ 1], sm.lse2[buf ^ 1], tid);
-      fence_proxy_async_smem();
-    }
+  int issued = 0;  // MMAs issued (chunk index of the next one)
+  auto issue = [&](int ch) {  // issuer only: Z^T of chunk ch into buffer ch % 2
+    const uint32_t qaddr = smem_addr(sm.qs[ch % QS]);
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk)
+      mma_ss(tmem + (ch & 1) * 128, sdesc_sw128(smem_addr(sm.k) + kk * 32),
+             sdesc_sw128(qaddr + kk * 32), IDESC, kk > 0);
+    mma_commit(b_mma[ch & 1]);
+  };
+  bool stop = false;
+  for (int g0 = 0; g0 < nchunks && !stop; g0 += QS) {
+    const int g1 = min(nchunks, g0 + QS);
+    // every MMA that read the chunk buffers has completed (waited below)
+    for (int ch = g0; ch < g1; ++ch) gather_chunk(p, h, ch, sm.qs[ch % QS], sm.lse2[ch % QS], tid);
+    cp_async_wait_all();
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
-    if (elected && ch + 1 < nchunks) {
+    if (issuer) {
       tc_fence_after();
-      if (k_ok) {
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          mma_ss(tmem + (buf ^ 1) * 128, sdesc_sw128(smem_addr(sm.k) + kk * 32),
-                 sdesc_sw128(smem_addr(sm.qs[buf ^ 1]) + kk * 32), IDESC, kk > 0);
+      if (g0 == 0) k_ok = mbar_wait(b_k, 0, abort_flag, WAIT_NS);
+      for (; issued < min(g1, g0 + 2); ++issued) {
+        if (k_ok) issue(issued);
+        else mma_commit(b_mma[issued & 1]);
       }
-      mma_commit(b_mma[buf ^ 1]);
     }
-    tc_fence_after();
-    uint32_t z[128];
-    tmem_ld128(tmem + lane_off + buf * 128, z);
-    const float* l2 = sm.lse2[buf];
-    float a4[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int ch = g0; ch < g1; ++ch) {
+      const int tb = ch & 1;
+      const bool ok = mbar_wait(b_mma[tb], ph[tb], abort_flag, WAIT_NS);
+      ph[tb] ^= 1;
+      tc_fence_after();
+      uint32_t z[128];
+      if (ok) tmem_ld128(tmem + lane_off + tb * 128, z);
+      tc_fence_before();
+      // every thread has read Z^T(ch): its buffer can take chunk ch+2
+      if (__syncthreads_or(!ok || *abort_flag)) {
+        stop = true;
+        break;
+      }
+      if (issuer && issued < g1) {
+        tc_fence_after();
+        if (k_ok) issue(issued);
+        else mma_commit(b_mma[issued & 1]);
+        ++issued;
+      }
+      const float* l2 = sm.lse2[ch % QS];
+      float a4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int i = 0; i < 128; ++i) a4[i & 3] += ex2(fmaf(__uint_as_float(z[i]), p.c, -l2[i]));
-    acc += (a4[0] + a4[1]) + (a4[2] + a4[3]);
+      for (int i = 0; i < 128; ++i) a4[i & 3] += ex2(fmaf(__uint_as_float(z[i]), p.c, -l2[i]));
+      acc += (a4[0] + a4[1]) + (a4[2] + a4[3]);
+    }
+    __syncthreads();  // lse2 and the chunk buffers are refilled by the next group
   }
   const int j = kt * BT + tid;
   if (j < p.N && !*abort_flag) p.sal[(size_t)h * p.N + j] = acc;
-  if (elected) {
+  if (issuer) {
     mma_commit(b_fin);
     mbar_wait(b_fin, 0, never, DRAIN_NS);
-    if (!k_ok) mbar_wait(b_k, 0, never, DRAIN_NS);
+    if (!k_ok || nchunks == 0) mbar_wait(b_k, 0, never, DRAIN_NS);
   }
+  cp_async_wait_all();
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {

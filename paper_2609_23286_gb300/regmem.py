@@ -53,7 +53,7 @@ class FrameDesc(ctypes.Structure):
 
 class Profile(ctypes.Structure):
     """regmem_profile."""
-    _fields_ = [("launches_attention", ctypes.c_int64), ("launches_combine", ctypes.c_int64),
+    _fields_ = [("launches_attention", ctypes.c_int64),
                 ("launches_saliency", ctypes.c_int64), ("launches_admit", ctypes.c_int64),
                 ("launches_anchor", ctypes.c_int64), ("attention_timed", ctypes.c_int64),
                 ("attention_ms", ctypes.c_double), ("attention_flops", ctypes.c_double),
@@ -64,8 +64,8 @@ class Profile(ctypes.Structure):
         return {f: getattr(self, f) for f, _ in self._fields_}
 
     def launches(self):
-        return (self.launches_attention + self.launches_combine + self.launches_saliency
-                + self.launches_admit + self.launches_anchor)
+        return (self.launches_attention + self.launches_saliency + self.launches_admit
+                + self.launches_anchor)
 
 
 class RegmemError(RuntimeError):

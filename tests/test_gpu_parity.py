@@ -263,3 +263,45 @@ def test_state_machine_and_argument_errors():
     with pytest.raises(regmem.RegmemError) as e:
         regmem.regmem_create(1, 1, 128, 1)
     assert e.value.status == regmem.ERR_UNSUPPORTED
+
+
+def test_uniform_keys_tie_to_lowest_indices():
+    """K = 0 makes every logit 0: softmax is uniform over the L attended keys,
+    every frame key has saliency |Q~| / L, and the admitted tokens must be the
+    k lowest candidate indices (ties go to the lower index)."""
+    H, ns, gh, gw, k = 4, 5, 8, 8, 20
+    N = ns + gh * gw
+    st = Stream(1, H, ns, gh, gw, budget=k, max_frames=3, seed=12)
+    try:
+        for t in (1, 2):
+            q, kk, v = st.inputs(0, t)
+            out, sal, lse = st.attend(0, q, torch.zeros_like(kk), v)
+            idx = st.admit(0, k)
+            torch.cuda.synchronize()
+            L = N if t == 1 else 2 * N
+            assert torch.allclose(lse.cpu().double(), torch.full((H, N), math.log(L), dtype=torch.float64),
+                                  atol=1e-4)
+            s_ref = np.full((H, N), 16.0 / L)
+            check_saliency(sal, s_ref, f"t={t}")
+            if t == 2:
+                assert (idx.cpu().numpy() == np.arange(ns, ns + k)[None, :]).all()
+    finally:
+        st.close()
+
+
+def test_admit_every_candidate():
+    """k equal to the number of candidates admits every patch token in order."""
+    H, ns, gh, gw = 2, 5, 8, 8
+    nc = gh * gw
+    st = Stream(1, H, ns, gh, gw, budget=nc, max_frames=3, seed=13)
+    try:
+        for t in (1, 2):
+            q, kk, v = st.inputs(0, t)
+            st.attend(0, q, kk, v)
+            idx = st.admit(0, nc)
+        torch.cuda.synchronize()
+        assert (idx.cpu().numpy() == np.arange(ns, ns + nc)[None, :]).all()
+        bk, bv = st.export(0)
+        assert torch.equal(bk[:, ns + gh * gw + 0:], kk[ns:, :, :].permute(1, 0, 2).cpu())
+    finally:
+        st.close()
