@@ -368,29 +368,10 @@ __global__ void __launch_bounds__(THREADS, 1)
           l *= alpha;
           m_used = mnew;
         }
-        // p = exp2(z * c - m_used): packed FMA for the argument, MUFU exp2,
-        // packed ADD for the row sum (two pair accumulators), bf16x2 pack.
-        const uint64_t cc = f2_pack(c, c), nn = f2_pack(-m_used, -m_used);
-        uint64_t acc2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
-        uint32_t pk[64];
-#pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          float a0, a1;
-          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[2 * i]), __uint_as_float(sr[2 * i + 1])), cc, nn),
-                    a0, a1);
-          const float p0 = ex2(a0), p1 = ex2(a1);
-          acc2[i & 1] = f2_add(acc2[i & 1], f2_pack(p0, p1));
-          pk[i] = pack_bf16x2(p0, p1);
-        }
-        {
-          float s0, s1, s2, s3;
-          f2_unpack(acc2[0], s0, s1);
-          f2_unpack(acc2[1], s2, s3);
-          l += (s0 + s1) + (s2 + s3);
-        }
         if (jj > 0) {
           // P V of the previous key tile must be done before P is overwritten
-          // and O is rescaled.
+          // and O is rescaled (it normally is by now: it was issued before S
+          // of this tile was read).
           ok = mbar_wait(b_odone, o_phase, abort_flag, WAIT_NS);
           o_phase ^= 1;
           if (__any_sync(0xffffffffu, !ok || *abort_flag)) {
@@ -399,11 +380,30 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           tc_fence_after();
         }
-        {  // P row -> TMEM (the A operand of the P V MMA)
-          uint32_t (&pa)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pk[0]);
-          uint32_t (&pb)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pk[32]);
-          tmem_st32(tm_p, pa);
-          tmem_st32(tm_p + 32, pb);
+        // p = exp2(z * c - m_used): packed FMA for the argument, MUFU exp2,
+        // packed ADD for the row sum, bf16x2 pack; P goes to TMEM in two
+        // 32-column halves so only half of it is held in registers.
+        const uint64_t cc = f2_pack(c, c), nn = f2_pack(-m_used, -m_used);
+        uint64_t acc2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int e = hf * 64 + 2 * i;
+            float a0, a1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), cc, nn), a0, a1);
+            const float p0 = ex2(a0), p1 = ex2(a1);
+            acc2[i & 1] = f2_add(acc2[i & 1], f2_pack(p0, p1));
+            pk[i] = pack_bf16x2(p0, p1);
+          }
+          tmem_st32(tm_p + 32 * hf, pk);
+        }
+        {
+          float s0, s1, s2, s3;
+          f2_unpack(acc2[0], s0, s1);
+          f2_unpack(acc2[1], s2, s3);
+          l += (s0 + s1) + (s2 + s3);
         }
         if (jj > 0 && __any_sync(0xffffffffu, need)) {  // rare: the max grew by > 2^8
           uint32_t orr[64];
