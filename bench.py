@@ -59,9 +59,14 @@ CONFIGS = {
 }
 
 # dram__bytes_read.sum + dram__bytes_write.sum of one attention-kernel launch,
-# from an ncu capture, scaled to the bench workload's mean launch; None until
-# a capture of the current kernel exists.
-ATTN_TRAFFIC_BYTES_PER_LAUNCH = None
+# from an ncu capture of the launch at the stream's mean attended length
+# (frame 1001 of the 2000-frame stream, L = 16,734: 72.49 MB read + 3.97 MB
+# written).  Set back to None whenever the
+# attention kernel changes until it is captured again.
+ATTN_TRAFFIC_BYTES_PER_LAUNCH = 76.46e6
+ATTN_TRAFFIC_NOTE = ("ncu dram bytes of the frame-1001 launch (mean attended length of the "
+                     "stream); the frame-2000 launch moves 554.7 MB (L2 no longer holds a "
+                     "layer's bank)")
 
 
 def describe(cfg, name):
@@ -459,6 +464,7 @@ def gpu_arm(args, cfg, cfg_name):
             "frac_of_burst_peak": round(attn_tflops / peak_burst, 4) if peak_burst else None,
             "peak_source": peak_src,
             "traffic": ATTN_TRAFFIC_BYTES_PER_LAUNCH,
+            "traffic_note": ATTN_TRAFFIC_NOTE if ATTN_TRAFFIC_BYTES_PER_LAUNCH else None,
             "launches": prof.attention_timed,
             "ctas": prof.attention_ctas,
             "ctas_per_sm": prof.attention_ctas_per_sm,
