@@ -24,14 +24,16 @@
 // then resets the counter.  CTAs wait on one another, so the kernel is
 // launched cooperatively (all CTAs resident, one per SM).
 //
-// CTA layout, warp-specialised (11 warps):
+// CTA layout, warp-specialised (12 warps, three warpgroups):
 //   warp 0       TMA producer: both Q tiles of a unit, then K and V tiles
 //                through separate 5-stage rings
 //   warps 1, 2   MMA issuers, one lane each, for query tile 0 and 1 (each
 //                follows only its own warpgroup's hand-offs, so a slower
 //                warpgroup never holds up the other's MMAs); warp 1 owns TMEM
-//   warps 3..6   softmax warpgroup 0 -> query tile 0 of the unit
-//   warps 7..10  softmax warpgroup 1 -> query tile 1 of the unit
+//   warp 3       idle (completes the control warpgroup, whose register
+//                budget is handed to the softmax warpgroups)
+//   warps 4..7   softmax warpgroup 0 -> query tile 0 of the unit
+//   warps 8..11  softmax warpgroup 1 -> query tile 1 of the unit
 // Each softmax thread owns one query row (its TMEM lane).  Each key tile is
 // loaded once and serves both query tiles.
 // TMEM (512 columns): S0 [0,128), S1 [128,256) fp32 logits; P0 [256,320),
@@ -40,14 +42,17 @@
 // P V is a TS-MMA (P from TMEM, V MN-major in smem).  Keeping P in TMEM keeps
 // it off shared memory, whose bandwidth the SS-MMA operand reads and the TMA
 // writes already use up.
-// Hand-offs are mbarriers: s_full (MMA -> softmax, per Q K^T), s_free
-// (softmax -> MMA, S consumed), p_ready (softmax -> MMA, P stored and O
-// rescaled), o_done (MMA -> softmax, per P V), K/V full and empty rings and
-// Q full/empty; the empty barriers take one arrival per issuer, and both
-// issuers wait every phase of the full barriers in order.  Each issuer
-// issues Q K^T of the next key tile as soon as S is consumed, so the tensor
-// core computes S(t+1) while the softmax of tile t runs, and the two query
-// tiles interleave on the tensor core.
+// Hand-offs are mbarriers: s_full (MMA -> softmax, S(j) computed), p_ready
+// (softmax -> MMA, P(j) stored and S(j) read), o_done (MMA -> softmax, P V(j)
+// done), K/V full and empty rings and Q full/empty; the empty barriers take
+// one arrival per issuer, and both issuers wait every phase of the full
+// barriers in order.  On GB300 each mbarrier hand-off costs a few hundred
+// cycles of latency (arrive, fence and a fresh wait alike), so a query tile
+// has three per key tile: the softmax waits for S(j), waits for P V(j-1)
+// before overwriting P, and arrives once P(j) is stored.  On that arrival the
+// issuer issues Q K^T(j+1) first (S(j) has been read) and then P V(j); the
+// softmax of the other query tile runs while the tensor core works for this
+// one, so the two warpgroups alternate instead of running in lockstep.
 // The softmax uses packed fp32x2 FMA/ADD and three-input max, leaving the
 // exp2 (MUFU) as the dominant instruction stream.
 // The softmax keeps a stale running max and only rescales O when the max
@@ -67,7 +72,12 @@ constexpr int BM = kTile, BN = kTile, HD = kHeadDim;
 constexpr int UROWS = kUnitRows;         // query rows per unit (two tiles)
 constexpr int KSTAGES = 5, VSTAGES = 5;
 constexpr int TILE_BYTES = BM * HD * 2;  // 16 KB bf16 tile
-constexpr int THREADS = 352;
+constexpr int THREADS = 384;
+// Register split: launched at 168 per thread (384 x 168 = 64,512); the
+// control warpgroup drops to 56 and the two softmax warpgroups rise to 224,
+// 128 x 56 + 256 x 224 = 64,512, the launch total.
+constexpr uint32_t REGS_CTRL = 56, REGS_SOFTMAX = 224;
+static_assert(128 * REGS_CTRL + 256 * REGS_SOFTMAX <= THREADS * 168, "register split");
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t TM_S0 = 0, TM_S1 = 128, TM_P0 = 256, TM_P1 = 320, TM_O0 = 384, TM_O1 = 448;
 constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s: a hung pipeline gives up
@@ -82,7 +92,7 @@ struct Smem {
   uint8_t v[VSTAGES][TILE_BYTES];
   uint64_t q_full, q_empty;
   uint64_t k_full[KSTAGES], k_empty[KSTAGES], v_full[VSTAGES], v_empty[VSTAGES];
-  uint64_t s_full[2], s_free[2], p_ready[2], o_done[2];
+  uint64_t s_full[2], p_ready[2], o_done[2];  // per query tile
   uint64_t fin_bar;
   uint32_t tmem_base;
   int abort_flag;
@@ -169,8 +179,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int t = 0; t < 2; ++t) {
       mbar_init(smem_addr(&sm.s_full[t]), 1);
-      mbar_init(smem_addr(&sm.s_free[t]), BM);
-      mbar_init(smem_addr(&sm.p_ready[t]), BM);
+      mbar_init(smem_addr(&sm.p_ready[t]), BM);  // every softmax thread arrives
       mbar_init(smem_addr(&sm.o_done[t]), 1);
     }
     mbar_init(smem_addr(&sm.fin_bar), 2);
@@ -185,7 +194,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
 
-  if (warp == 0) {
+  if (warp < 4) {
+   setmaxnreg_dec<REGS_CTRL>();
+   if (warp == 0) {
     // ================================================================ producer
     if (lane == 0) {
       prefetch_tmap(&tmQ);
@@ -241,9 +252,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t sq = smem_addr(sm.q[t]);
       const uint32_t d_s = tmem + (t ? TM_S1 : TM_S0), d_p = tmem + (t ? TM_P1 : TM_P0);
       const uint32_t d_o = tmem + (t ? TM_O1 : TM_O0);
-      const uint32_t b_sfull = smem_addr(&sm.s_full[t]), b_sfree = smem_addr(&sm.s_free[t]);
-      const uint32_t b_pready = smem_addr(&sm.p_ready[t]), b_odone = smem_addr(&sm.o_done[t]);
-      int nqk = 0, npv = 0;  // Q K^T / P V issued for this query tile
+      const uint32_t b_sfull = smem_addr(&sm.s_full[t]), b_pready = smem_addr(&sm.p_ready[t]);
+      const uint32_t b_odone = smem_addr(&sm.o_done[t]);
+      int npv = 0;  // P V issued for this query tile (= p_ready phases consumed)
       int it = 0, piece = 0;
       bool ok = true;
       for (long long x = x_begin; x < x_end && ok;) {
@@ -263,35 +274,42 @@ __global__ void __launch_bounds__(THREADS, 1)
         ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, WAIT_NS);
         const int t0 = it;  // CTA-local index of the piece's first key tile
         it += n;
-        // Step jj issues Q K^T of tile jj+1 (as soon as S is free) and then
-        // P V of tile jj (once P is stored); step -1 is the prologue.
-        for (int jj = -1; jj < n && ok; ++jj) {
-          if (jj + 1 < n) {
-            const int tq = t0 + jj + 1;
-            const int ks = tq % KSTAGES;
-            ok = mbar_wait(smem_addr(&sm.k_full[ks]), (tq / KSTAGES) & 1, abort_flag, WAIT_NS);
-            if (ok && act && nqk > 0) ok = mbar_wait(b_sfree, (nqk - 1) & 1, abort_flag, WAIT_NS);
-            if (!ok) break;
-            if (act) {
-              tc_fence_after();
-              const uint32_t kaddr = smem_addr(sm.k[ks]);
+        // Q K^T of key tile jj of the piece into S; its K stage (and, after the
+        // piece's last one, the Q tiles) are released when the MMAs complete.
+        auto issue_qk = [&](int jj) {
+          const int ks = (t0 + jj) % KSTAGES;
+          if (act) {
+            const uint32_t kaddr = smem_addr(sm.k[ks]);
 #pragma unroll
-              for (int kk = 0; kk < HD / 16; ++kk)
-                mma_ss(d_s, sdesc_sw128(sq + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
-              mma_commit(b_sfull);
-              ++nqk;
-            }
-            release(smem_addr(&sm.k_empty[ks]));
-            if (jj + 2 == n) release(smem_addr(&sm.q_empty));
+            for (int kk = 0; kk < HD / 16; ++kk)
+              mma_ss(d_s, sdesc_sw128(sq + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
+            mma_commit(b_sfull);
           }
-          if (jj < 0) continue;
+          release(smem_addr(&sm.k_empty[ks]));
+          if (jj + 1 == n) release(smem_addr(&sm.q_empty));
+        };
+        auto wait_k = [&](int jj) {
+          const int tq = t0 + jj;
+          return mbar_wait(smem_addr(&sm.k_full[tq % KSTAGES]), (tq / KSTAGES) & 1, abort_flag, WAIT_NS);
+        };
+        if (ok) ok = wait_k(0);
+        if (ok) {
+          tc_fence_after();
+          issue_qk(0);
+        }
+        // Step jj: once P(jj) is stored (which also means S(jj) has been read),
+        // Q K^T of tile jj+1 goes first, so that the softmax gets its next S
+        // early, then P V of tile jj.
+        for (int jj = 0; jj < n && ok; ++jj) {
           const int tp = t0 + jj;
           const int vs = tp % VSTAGES;
-          ok = mbar_wait(smem_addr(&sm.v_full[vs]), (tp / VSTAGES) & 1, abort_flag, WAIT_NS);
+          if (jj + 1 < n) ok = wait_k(jj + 1);
+          if (ok) ok = mbar_wait(smem_addr(&sm.v_full[vs]), (tp / VSTAGES) & 1, abort_flag, WAIT_NS);
           if (ok && act) ok = mbar_wait(b_pready, npv & 1, abort_flag, WAIT_NS);
           if (!ok) break;
+          tc_fence_after();
+          if (jj + 1 < n) issue_qk(jj + 1);
           if (act) {
-            tc_fence_after();
             const uint32_t vaddr = smem_addr(sm.v[vs]);
 #pragma unroll
             for (int kk = 0; kk < BN / 16; ++kk)  // 16 keys = 8 packed columns of P
@@ -307,20 +325,33 @@ __global__ void __launch_bounds__(THREADS, 1)
       mma_commit(smem_addr(&sm.fin_bar));
       mbar_wait(smem_addr(&sm.fin_bar), 0, never, DRAIN_NS);
     }
+   }
   } else {
+    setmaxnreg_inc<REGS_SOFTMAX>();
     // ================================================================ softmax
-    const int t = (warp - 3) >> 2;          // query tile of this warpgroup
+    const int t = (warp - 4) >> 2;          // query tile of this warpgroup
     const int quarter = warp & 3;           // TMEM lane quarter of this warp
     const int row = quarter * 32 + lane;    // query row inside the tile
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
     const uint32_t tm_s = tmem + lane_off + (t ? TM_S1 : TM_S0);
     const uint32_t tm_o = tmem + lane_off + (t ? TM_O1 : TM_O0);
-    const uint32_t b_sfull = smem_addr(&sm.s_full[t]), b_sfree = smem_addr(&sm.s_free[t]);
-    const uint32_t b_pready = smem_addr(&sm.p_ready[t]), b_odone = smem_addr(&sm.o_done[t]);
+    const uint32_t b_sfull = smem_addr(&sm.s_full[t]), b_pready = smem_addr(&sm.p_ready[t]);
+    const uint32_t b_odone = smem_addr(&sm.o_done[t]);
     const uint32_t tm_p = tmem + lane_off + (t ? TM_P1 : TM_P0);
     const float c = p.scale_log2;
     uint32_t s_phase = 0, o_phase = 0;
     bool stop = false;
+    // Waits for a phase; the result is uniform across the warp.
+    auto wait_phase = [&](uint32_t bar, uint32_t parity) -> bool {
+      const bool ok = mbar_wait(bar, parity, abort_flag, WAIT_NS);
+      if (__any_sync(0xffffffffu, !ok)) return false;
+      tc_fence_after();
+      return true;
+    };
+    // Per key tile the warpgroup has three hand-offs: it waits for S(j), waits
+    // for P V(j-1) (P is single-buffered), and arrives once P(j) is stored,
+    // which also tells the issuer that S(j) has been read.  Every thread
+    // arrives (cheaper than a warp-elected arrival after a warp barrier).
     for (long long x = x_begin; x < x_end && !stop;) {
       const Piece pc = piece_at(p, x, x_end);
       const int n = pc.j1 - pc.j0;
@@ -330,17 +361,13 @@ __global__ void __launch_bounds__(THREADS, 1)
       float l = 0.f;             // running row sum of exp2(z*c - m_used)
       for (int jj = 0; jj < n; ++jj) {
         const int j = pc.j0 + jj;
-        bool ok = mbar_wait(b_sfull, s_phase, abort_flag, WAIT_NS);  // S(j) in TMEM
-        s_phase ^= 1;
-        if (__any_sync(0xffffffffu, !ok || *abort_flag)) {
+        if (!wait_phase(b_sfull, s_phase)) {  // S(j) in TMEM
           stop = true;
           break;
         }
-        tc_fence_after();
+        s_phase ^= 1;
         uint32_t sr[128];
         tmem_ld128(tm_s, sr);
-        tc_fence_before();
-        mbar_arrive(b_sfree);  // S consumed: the next Q K^T may overwrite it
         const int valid = tile_valid(p, j);
         if (valid < BN) {
 #pragma unroll
@@ -368,26 +395,14 @@ __global__ void __launch_bounds__(THREADS, 1)
           l *= alpha;
           m_used = mnew;
         }
-        if (jj > 0) {
-          // P V of the previous key tile must be done before P is overwritten
-          // and O is rescaled (it normally is by now: it was issued before S
-          // of this tile was read).
-          ok = mbar_wait(b_odone, o_phase, abort_flag, WAIT_NS);
-          o_phase ^= 1;
-          if (__any_sync(0xffffffffu, !ok || *abort_flag)) {
-            stop = true;
-            break;
-          }
-          tc_fence_after();
-        }
         // p = exp2(z * c - m_used): packed FMA for the argument, MUFU exp2,
-        // packed ADD for the row sum, bf16x2 pack; P goes to TMEM in two
-        // 32-column halves so only half of it is held in registers.
+        // packed ADD for the row sum, bf16x2 pack.  P is computed in registers
+        // before its TMEM columns are known to be free.
         const uint64_t cc = f2_pack(c, c), nn = f2_pack(-m_used, -m_used);
         uint64_t acc2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
+        uint32_t pk[2][32];
 #pragma unroll
         for (int hf = 0; hf < 2; ++hf) {
-          uint32_t pk[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             const int e = hf * 64 + 2 * i;
@@ -395,38 +410,47 @@ __global__ void __launch_bounds__(THREADS, 1)
             f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), cc, nn), a0, a1);
             const float p0 = ex2(a0), p1 = ex2(a1);
             acc2[i & 1] = f2_add(acc2[i & 1], f2_pack(p0, p1));
-            pk[i] = pack_bf16x2(p0, p1);
+            pk[hf][i] = pack_bf16x2(p0, p1);
           }
-          tmem_st32(tm_p + 32 * hf, pk);
         }
+        if (jj > 0) {
+          // P V(j-1) has read P and added into O
+          if (!wait_phase(b_odone, o_phase)) {
+            stop = true;
+            break;
+          }
+          o_phase ^= 1;
+          if (__any_sync(0xffffffffu, need)) {
+            // rare (the max grew by > 2^8): rescale O before P V(j) adds to it
+#pragma unroll 1
+            for (int hc = 0; hc < 2; ++hc) {  // 32 columns at a time
+              uint32_t orr[32];
+              tmem_ld32(tm_o + 32 * hc, orr);
+#pragma unroll
+              for (int i = 0; i < 32; ++i) orr[i] = __float_as_uint(__uint_as_float(orr[i]) * alpha);
+              tmem_st32(tm_o + 32 * hc, orr);
+            }
+          }
+        }
+        tmem_st32_async(tm_p, pk[0]);
+        tmem_st32_async(tm_p + 32, pk[1]);
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(b_pready);
         {
           float s0, s1, s2, s3;
           f2_unpack(acc2[0], s0, s1);
           f2_unpack(acc2[1], s2, s3);
           l += (s0 + s1) + (s2 + s3);
         }
-        if (jj > 0 && __any_sync(0xffffffffu, need)) {  // rare: the max grew by > 2^8
-          uint32_t orr[64];
-          tmem_ld64(tm_o, orr);
-#pragma unroll
-          for (int i = 0; i < 64; ++i) orr[i] = __float_as_uint(__uint_as_float(orr[i]) * alpha);
-          uint32_t (&oa)[32] = *reinterpret_cast<uint32_t(*)[32]>(&orr[0]);
-          uint32_t (&ob)[32] = *reinterpret_cast<uint32_t(*)[32]>(&orr[32]);
-          tmem_st32(tm_o, oa);
-          tmem_st32(tm_o + 32, ob);
-        }
-        tc_fence_before();
-        mbar_arrive(b_pready);
       }
       if (stop) break;
       // -------------------------------------------------------------- epilogue
-      const bool ok = mbar_wait(b_odone, o_phase, abort_flag, WAIT_NS);
-      o_phase ^= 1;
-      if (__any_sync(0xffffffffu, !ok || *abort_flag)) {
+      if (!wait_phase(b_odone, o_phase)) {  // the last tile's P V
         stop = true;
         break;
       }
-      tc_fence_after();
+      o_phase ^= 1;
       uint32_t orr[64];
       tmem_ld64(tm_o, orr);
       tc_fence_before();
@@ -491,19 +515,23 @@ __global__ void __launch_bounds__(THREADS, 1)
             const size_t pr = (size_t)bb * UROWS + t * BM + row;
             const float lp = __ldcg(p.part_lse + pr);
             const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD);
-            float4 v[16];
-#pragma unroll
-            for (int c4 = 0; c4 < 16; ++c4) v[c4] = __ldcg(src + c4);
             const float mn = fmaxf(m, lp);
             const float a_old = ex2((m - mn) * 1.4426950408889634f);
             const float a_new = ex2((lp - mn) * 1.4426950408889634f);
             den = den * a_old + a_new;
 #pragma unroll
-            for (int c4 = 0; c4 < 16; ++c4) {
-              acc[c4 * 4 + 0] = acc[c4 * 4 + 0] * a_old + v[c4].x * a_new;
-              acc[c4 * 4 + 1] = acc[c4 * 4 + 1] * a_old + v[c4].y * a_new;
-              acc[c4 * 4 + 2] = acc[c4 * 4 + 2] * a_old + v[c4].z * a_new;
-              acc[c4 * 4 + 3] = acc[c4 * 4 + 3] * a_old + v[c4].w * a_new;
+            for (int g = 0; g < 4; ++g) {  // 16 columns at a time
+              float4 v[4];
+#pragma unroll
+              for (int c4 = 0; c4 < 4; ++c4) v[c4] = __ldcg(src + g * 4 + c4);
+#pragma unroll
+              for (int c4 = 0; c4 < 4; ++c4) {
+                const int e = (g * 4 + c4) * 4;
+                acc[e + 0] = acc[e + 0] * a_old + v[c4].x * a_new;
+                acc[e + 1] = acc[e + 1] * a_old + v[c4].y * a_new;
+                acc[e + 2] = acc[e + 2] * a_old + v[c4].z * a_new;
+                acc[e + 3] = acc[e + 3] * a_old + v[c4].w * a_new;
+              }
             }
             m = mn;
           }
