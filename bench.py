@@ -3,7 +3,9 @@
 
 A step is one frame through every global-attention layer: per layer, the
 regulated attention over [memory ; frame] with LSE (Eq. 3), the LSE-saliency
-(Sec. 3.3) and the top-k admission into the layer's bank (Eq. 4 / Eq. 6).
+(Sec. 3.3) and the top-k admission into the layer's bank (Eq. 4 / Eq. 6),
+issued as one regmem_attend_admit call per layer (the admission runs inside
+the saliency kernel).
 Default workload: the long-horizon stream -- 24 layers, 16 heads x 64,
 1374 tokens per frame (37x37 patches + 5 special tokens), k = 14 admitted
 rows per head per frame, 2000 frames, so each layer's memory grows from 0 to
@@ -18,7 +20,7 @@ needed.
 Also reported:
   roofline      attention kernel: algorithmic FLOPs / CUDA-event time of its
                 launches in the timed region, against the measured bf16 peak
-  e2e           same metric through regmem_attend_frame_host: pinned host
+  e2e           same metric through regmem_attend_admit_host: pinned host
                 Q/K/V in, O and saliency back to host, copies inside the timed
                 region
   cpu_baseline  the fp64 oracle on the host cores, timed on a bounded sample
@@ -282,8 +284,9 @@ def make_pool(cfg, P, seed, device):
     return pool
 
 
-def run_frames(rm, cfg, pool, t0, count, out, sal, fa_out=None):
-    """Enqueue frames t0 .. t0+count-1 (all layers) through the C ABI."""
+def run_frames(rm, cfg, pool, t0, count, out, sal, fa_out=None, two_call=False):
+    """Enqueue frames t0 .. t0+count-1 (all layers) through the C ABI: one
+    regmem_attend_admit per layer, or regmem_attend_frame + regmem_admit."""
     P = len(pool[0])
     for t in range(t0, t0 + count):
         for layer in range(cfg["layers"]):
@@ -291,8 +294,11 @@ def run_frames(rm, cfg, pool, t0, count, out, sal, fa_out=None):
             if fa_out is not None:
                 fq, fk, fv = pool[layer][t % P]
                 rm.frame_attention(fq, fk, fv, fa_out)
-            rm.attend_frame(layer, q, k, v, out, sal)
-            rm.admit(layer, cfg["k"])
+            if two_call:
+                rm.attend_frame(layer, q, k, v, out, sal)
+                rm.admit(layer, cfg["k"])
+            else:
+                rm.attend_admit(layer, q, k, v, out, sal, cfg["k"])
 
 
 def synthetic_bank(cfg, rows, seed, device):
@@ -355,7 +361,7 @@ def gpu_arm(args, cfg, cfg_name):
 
     # warm-up frames, then a fresh stream (or the restored late-stream banks)
     restore()
-    run_frames(rm, cfg, pool, S0, W, out, sal, fa_out)
+    run_frames(rm, cfg, pool, S0, W, out, sal, fa_out, args.two_call)
     rm.synchronize()
     restore()
 
@@ -366,7 +372,7 @@ def gpu_arm(args, cfg, cfg_name):
     torch.cuda.synchronize()
     clocks.start()
     ev0.record(stream)
-    run_frames(rm, cfg, pool, S0, K, out, sal, fa_out)
+    run_frames(rm, cfg, pool, S0, K, out, sal, fa_out, args.two_call)
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -397,8 +403,7 @@ def gpu_arm(args, cfg, cfg_name):
                 if hfa is not None:
                     fq, fk, fv = pool[layer][t % P]
                     rm.frame_attention(fq, fk, fv, fa_out)  # frame-attention layer: device inputs
-                rm.attend_frame_host(layer, q, k, v, hout, hsal)
-                rm.admit(layer, cfg["k"])
+                rm.attend_admit_host(layer, q, k, v, hout, hsal, cfg["k"])
         e1.record(stream)
         rm.synchronize()
         barrier()
@@ -406,7 +411,7 @@ def gpu_arm(args, cfg, cfg_name):
         tb = N * H * 64 * 2
         e2e = {"value": round(K * world / (e2e_ms / 1e3), 3), "unit": UNIT,
                "h2d_bytes_per_step": 3 * tb * L, "d2h_bytes_per_step": (tb + H * N * 4) * L,
-               "api": "regmem_attend_frame_host + regmem_admit (pinned host buffers)"}
+               "api": "regmem_attend_admit_host (pinned host buffers)"}
 
     launches = int(sum_over_ranks(prof.launches(), dev))
     rm.close()
@@ -530,6 +535,8 @@ def main(argv=None):
     ap.add_argument("--layers", type=int, default=0, help="override the config's layer count")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--two-call", action="store_true",
+                    help="per layer regmem_attend_frame + regmem_admit instead of regmem_attend_admit")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be >= 3")

@@ -129,6 +129,27 @@ REGMEM_API regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, co
  * State: the layer must have an attend pending (ERR_STATE). */
 REGMEM_API regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out);
 
+/* regmem_attend_frame followed by regmem_admit(layer, k, idx_out), in one
+ * call: the whole per-frame step of one layer (Eq. 3, the LSE-Saliency of
+ * Sec. 3.3, then Eq. 4 or Eq. 6).  The admission runs inside the saliency
+ * kernel (the last block of each head selects and appends), so it needs no
+ * launch of its own.  Arguments, layouts, k range and errors as in the two
+ * calls; every check (including k and capacity) is made before anything is
+ * enqueued.  The library keeps no pointer after the call: K, V and saliency
+ * need only stay valid until the enqueued work has run.
+ * State: the layer must not have an attend pending (ERR_STATE); afterwards
+ * it has none. */
+REGMEM_API regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, const void* K,
+                                  const void* V, void* out, float* saliency, int32_t k,
+                                  int32_t* idx_out);
+
+/* regmem_attend_admit with HOST buffers (layouts and staging as in
+ * regmem_attend_frame_host; no index output).  The device->host copies of
+ * out and saliency are complete after regmem_synchronize. */
+REGMEM_API regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* hostQ,
+                                       const void* hostK, const void* hostV, void* hostOut,
+                                       float* hostSaliency, int32_t k);
+
 /* Non-causal attention inside one frame (the frame-attention layers that
  * alternate with the global ones, Sec. 3.1): out = softmax(Q K^T scale) V
  * over the frame's own N keys, no memory, no saliency.  Uses the geometry of

@@ -53,21 +53,6 @@ int attn_smem_bytes();                                 // dynamic shared memory 
 cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_before = nullptr,
                              cudaEvent_t ev_after = nullptr);
 
-// LSE-Saliency over the frame's own keys, per (head, 128-key tile).
-struct SalArgs {
-  const CUtensorMap* tmK;   // frame K map (same as the attention's)
-  const __nv_bfloat16* Q;   // [N][H][64]
-  const int* qidx;          // sampled query tokens, [nq]
-  int nq;
-  const float* lse;         // [H][N]
-  int N, H;
-  float scale;
-  float* sal;               // [H][N]
-  int* status;
-};
-cudaError_t saliency_setup();
-cudaError_t launch_saliency(const SalArgs& a, cudaStream_t s);
-
 // Per-head top-k of the candidates' saliency and append to the bank.
 struct AdmitArgs {
   const float* sal;         // [H][N]
@@ -79,6 +64,11 @@ struct AdmitArgs {
   long long M;              // rows already in the bank
   int N, H, cand_lo, k;
   int32_t* idx_out;         // optional [H][k]
+  // distributed selection (k <= 32): per-(head, 128-key tile) lists and
+  // per-head completion counters (zero between launches); null -> one block
+  // per head selects alone
+  uint64_t* lists;          // [H][ceil(N/128)][32]
+  int* done;                // [H]
 };
 cudaError_t admit_setup();
 cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s);
@@ -86,6 +76,26 @@ cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s);
 cudaError_t launch_anchor(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
                           __nv_bfloat16* bankV, long long cap, int N, int H, cudaStream_t s);
 
+// LSE-Saliency over the frame's own keys, per (head, 128-key tile).  With
+// `adm` set (1 <= k <= 32, sal == adm->sal, lists and done given), each block
+// also keeps its tile's best admission candidates and the last block to
+// finish a head runs that head's admission.
+struct SalArgs {
+  const CUtensorMap* tmK;   // frame K map (same as the attention's)
+  const __nv_bfloat16* Q;   // [N][H][64]
+  const int* qidx;          // sampled query tokens, [nq]
+  int nq;
+  const float* lse;         // [H][N]
+  int N, H;
+  float scale;
+  float* sal;               // [H][N]
+  int* status;
+  const AdmitArgs* adm;     // optional fused admission
+};
+cudaError_t saliency_setup();
+cudaError_t launch_saliency(const SalArgs& a, cudaStream_t s);
+
 constexpr int kMaxCandidates = 8192;
+constexpr int kFusedMaxK = 32;  // largest k of the distributed (list) selection
 
 }  // namespace regmem_dev

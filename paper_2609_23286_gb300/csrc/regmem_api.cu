@@ -43,6 +43,8 @@ struct regmem {
   float* part_o = nullptr;    // split-KV partials
   float* part_lse = nullptr;
   int* counters = nullptr;    // split-piece counters, [units][2]
+  int* head_done = nullptr;   // per-head completion counters of the distributed selection
+  uint64_t* adm_lists = nullptr;  // per-(head, key tile) candidate lists, [H][nkt][32]
   int attn_grid = 0;
   int attn_ctas_per_sm = 0;
   int* status_host = nullptr; // mapped pinned word written by kernels
@@ -309,6 +311,9 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   const size_t n_counters = (size_t)attn_plan(N, h->heads, 0).units * 2;
   RM_CUDA(h, cudaMalloc(&h->counters, n_counters * sizeof(int)));
   RM_CUDA(h, cudaMemset(h->counters, 0, n_counters * sizeof(int)));
+  RM_CUDA(h, cudaMalloc(&h->head_done, h->heads * sizeof(int)));
+  RM_CUDA(h, cudaMemset(h->head_done, 0, h->heads * sizeof(int)));
+  RM_CUDA(h, cudaMalloc(&h->adm_lists, (size_t)h->heads * ((N + kTile - 1) / kTile) * 32 * sizeof(uint64_t)));
   RM_CUDA(h, cudaHostAlloc(&h->status_host, sizeof(int), cudaHostAllocMapped));
   *h->status_host = 0;
   RM_CUDA(h, cudaHostGetDevicePointer(&h->status_dev, h->status_host, 0));
@@ -341,19 +346,14 @@ regmem_status regmem_set_stream(regmem_t* h, void* stream) {
   return REGMEM_OK;
 }
 
-regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, const void* K,
-                                  const void* V, void* out, float* saliency) {
-  regmem_status s = ready(h, layer, true);
-  if (s != REGMEM_OK) return s;
-  if (!Q || !K || !V || !out || !saliency)
-    return fail(h, REGMEM_ERR_ARG, "null tensor pointer");
-  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(out) || !aligned16(saliency))
-    return fail(h, REGMEM_ERR_ARG, "tensor pointers must be 16-byte aligned");
-  if (h->pending[layer])
-    return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
-                layer);
+namespace {
+
+// Attention and saliency of one frame on one layer; with `adm` the saliency
+// kernel also runs the admission of adm->k rows per head (fused path).
+regmem_status attend_impl(regmem_t* h, int32_t layer, const void* Q, const void* K, const void* V,
+                          void* out, float* saliency, const AdmitArgs* adm) {
   const long long M = h->len[layer];
-  s = run_attention(h, layer, Q, K, V, out, (int)M);
+  regmem_status s = run_attention(h, layer, Q, K, V, out, (int)M);
   if (s != REGMEM_OK) return s;
   CUtensorMap tk;
   if (!encode_frame_map(&tk, K, h->N, h->heads))
@@ -369,8 +369,65 @@ regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, con
   sa.scale = h->scale;
   sa.sal = saliency;
   sa.status = h->status_dev;
+  sa.adm = adm;
   RM_CUDA(h, launch_saliency(sa, h->stream));
   h->prof.launches_saliency += 1;
+  return REGMEM_OK;
+}
+
+regmem_status check_tensors(regmem_t* h, const void* Q, const void* K, const void* V,
+                            const void* out, const float* saliency) {
+  if (!Q || !K || !V || !out || !saliency)
+    return fail(h, REGMEM_ERR_ARG, "null tensor pointer");
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(out) || !aligned16(saliency))
+    return fail(h, REGMEM_ERR_ARG, "tensor pointers must be 16-byte aligned");
+  return REGMEM_OK;
+}
+
+// k range and capacity of an admission on a non-empty layer.
+regmem_status check_admit(regmem_t* h, int32_t layer, int32_t k) {
+  const int nc = h->N - h->cand_lo;
+  const int kmax = h->budget < nc ? h->budget : nc;
+  if (k < 0 || k > kmax)
+    return fail(h, REGMEM_ERR_ARG, "k = %d outside [0, %d] (budget %d, candidates %d)", k, kmax,
+                h->budget, nc);
+  if (h->len[layer] + k > h->cap)
+    return fail(h, REGMEM_ERR_CAPACITY, "layer %d: %lld + %d rows exceed capacity %lld", layer,
+                h->len[layer], k, h->cap);
+  return REGMEM_OK;
+}
+
+AdmitArgs admit_args(regmem_t* h, int32_t layer, const void* K, const void* V, float* saliency,
+                     int32_t k, int32_t* idx_out) {
+  AdmitArgs a;
+  a.sal = saliency;
+  a.K = static_cast<const __nv_bfloat16*>(K);
+  a.V = static_cast<const __nv_bfloat16*>(V);
+  a.bankK = h->bankK + (size_t)layer * h->heads * h->cap * kHeadDim;
+  a.bankV = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
+  a.cap = h->cap;
+  a.M = h->len[layer];
+  a.N = h->N;
+  a.H = h->heads;
+  a.cand_lo = h->cand_lo;
+  a.k = k;
+  a.idx_out = idx_out;
+  a.lists = h->adm_lists;
+  a.done = h->head_done;
+  return a;
+}
+
+}  // namespace
+
+regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, const void* K,
+                                  const void* V, void* out, float* saliency) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if ((s = check_tensors(h, Q, K, V, out, saliency)) != REGMEM_OK) return s;
+  if (h->pending[layer])
+    return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
+                layer);
+  if ((s = attend_impl(h, layer, Q, K, V, out, saliency, nullptr)) != REGMEM_OK) return s;
   h->pending[layer] = 1;
   h->pK[layer] = static_cast<const __nv_bfloat16*>(K);
   h->pV[layer] = static_cast<const __nv_bfloat16*>(V);
@@ -378,16 +435,47 @@ regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, con
   return REGMEM_OK;
 }
 
-regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* hostQ,
-                                       const void* hostK, const void* hostV, void* hostOut,
-                                       float* hostSaliency) {
+regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, const void* K,
+                                  const void* V, void* out, float* saliency, int32_t k,
+                                  int32_t* idx_out) {
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
-  if (!hostQ || !hostK || !hostV || !hostOut || !hostSaliency)
-    return fail(h, REGMEM_ERR_ARG, "null host pointer");
+  if ((s = check_tensors(h, Q, K, V, out, saliency)) != REGMEM_OK) return s;
   if (h->pending[layer])
     return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
                 layer);
+  if (idx_out && ((reinterpret_cast<uintptr_t>(idx_out) & 3u) != 0))
+    return fail(h, REGMEM_ERR_ARG, "idx_out must be 4-byte aligned");
+  if (h->len[layer] == 0) {  // Eq. 4: the first frame is kept whole
+    if ((s = attend_impl(h, layer, Q, K, V, out, saliency, nullptr)) != REGMEM_OK) return s;
+    auto* bk = h->bankK + (size_t)layer * h->heads * h->cap * kHeadDim;
+    auto* bv = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
+    RM_CUDA(h, launch_anchor(static_cast<const __nv_bfloat16*>(K), static_cast<const __nv_bfloat16*>(V),
+                             bk, bv, h->cap, h->N, h->heads, h->stream));
+    h->prof.launches_anchor += 1;
+    h->len[layer] = h->N;
+    return REGMEM_OK;
+  }
+  if ((s = check_admit(h, layer, k)) != REGMEM_OK) return s;
+  const AdmitArgs a = admit_args(h, layer, K, V, saliency, k, idx_out);
+  // k <= 32: the admission runs inside the saliency kernel; larger k takes
+  // the separate single-block selection
+  const bool fused = k > 0 && k <= kFusedMaxK;
+  if ((s = attend_impl(h, layer, Q, K, V, out, saliency, fused ? &a : nullptr)) != REGMEM_OK) return s;
+  if (k > 0 && !fused) {
+    RM_CUDA(h, launch_admit(a, h->stream));
+    h->prof.launches_admit += 1;
+  }
+  h->len[layer] += k;
+  return REGMEM_OK;
+}
+
+namespace {
+
+// Copies a frame's Q, K, V from host memory into the handle's staging buffers
+// (K and V per layer: they must stay valid until the layer's admission).
+regmem_status stage_inputs(regmem_t* h, int32_t layer, const void* hostQ, const void* hostK,
+                           const void* hostV) {
   const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
   const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
   if (!h->stQ) {
@@ -402,11 +490,51 @@ regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* h
   RM_CUDA(h, cudaMemcpyAsync(h->stQ, hostQ, tbytes, cudaMemcpyHostToDevice, h->stream));
   RM_CUDA(h, cudaMemcpyAsync(h->stK[layer], hostK, tbytes, cudaMemcpyHostToDevice, h->stream));
   RM_CUDA(h, cudaMemcpyAsync(h->stV[layer], hostV, tbytes, cudaMemcpyHostToDevice, h->stream));
-  s = regmem_attend_frame(h, layer, h->stQ, h->stK[layer], h->stV[layer], h->stOut, h->stSal);
-  if (s != REGMEM_OK) return s;
+  return REGMEM_OK;
+}
+
+regmem_status unstage_outputs(regmem_t* h, void* hostOut, float* hostSaliency) {
+  const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
+  const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
   RM_CUDA(h, cudaMemcpyAsync(hostOut, h->stOut, tbytes, cudaMemcpyDeviceToHost, h->stream));
   RM_CUDA(h, cudaMemcpyAsync(hostSaliency, h->stSal, sbytes, cudaMemcpyDeviceToHost, h->stream));
   return REGMEM_OK;
+}
+
+}  // namespace
+
+regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* hostQ,
+                                       const void* hostK, const void* hostV, void* hostOut,
+                                       float* hostSaliency) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if (!hostQ || !hostK || !hostV || !hostOut || !hostSaliency)
+    return fail(h, REGMEM_ERR_ARG, "null host pointer");
+  if (h->pending[layer])
+    return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
+                layer);
+  if ((s = stage_inputs(h, layer, hostQ, hostK, hostV)) != REGMEM_OK) return s;
+  s = regmem_attend_frame(h, layer, h->stQ, h->stK[layer], h->stV[layer], h->stOut, h->stSal);
+  if (s != REGMEM_OK) return s;
+  return unstage_outputs(h, hostOut, hostSaliency);
+}
+
+regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* hostQ,
+                                       const void* hostK, const void* hostV, void* hostOut,
+                                       float* hostSaliency, int32_t k) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if (!hostQ || !hostK || !hostV || !hostOut || !hostSaliency)
+    return fail(h, REGMEM_ERR_ARG, "null host pointer");
+  if (h->pending[layer])
+    return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
+                layer);
+  if (h->len[layer] > 0 && (s = check_admit(h, layer, k)) != REGMEM_OK) return s;
+  if ((s = stage_inputs(h, layer, hostQ, hostK, hostV)) != REGMEM_OK) return s;
+  s = regmem_attend_admit(h, layer, h->stQ, h->stK[layer], h->stV[layer], h->stOut, h->stSal, k,
+                          nullptr);
+  if (s != REGMEM_OK) return s;
+  return unstage_outputs(h, hostOut, hostSaliency);
 }
 
 regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out) {
@@ -416,37 +544,18 @@ regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_o
     return fail(h, REGMEM_ERR_STATE, "layer %d has no attend pending", layer);
   if (idx_out && ((reinterpret_cast<uintptr_t>(idx_out) & 3u) != 0))
     return fail(h, REGMEM_ERR_ARG, "idx_out must be 4-byte aligned");
-  auto* bk = h->bankK + (size_t)layer * h->heads * h->cap * kHeadDim;
-  auto* bv = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
   if (h->len[layer] == 0) {  // Eq. 4: the first frame is kept whole
+    auto* bk = h->bankK + (size_t)layer * h->heads * h->cap * kHeadDim;
+    auto* bv = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
     RM_CUDA(h, launch_anchor(h->pK[layer], h->pV[layer], bk, bv, h->cap, h->N, h->heads, h->stream));
     h->prof.launches_anchor += 1;
     h->len[layer] = h->N;
     h->pending[layer] = 0;
     return REGMEM_OK;
   }
-  const int nc = h->N - h->cand_lo;
-  const int kmax = h->budget < nc ? h->budget : nc;
-  if (k < 0 || k > kmax)
-    return fail(h, REGMEM_ERR_ARG, "k = %d outside [0, %d] (budget %d, candidates %d)", k, kmax,
-                h->budget, nc);
-  if (h->len[layer] + k > h->cap)
-    return fail(h, REGMEM_ERR_CAPACITY, "layer %d: %lld + %d rows exceed capacity %lld", layer,
-                h->len[layer], k, h->cap);
+  if ((s = check_admit(h, layer, k)) != REGMEM_OK) return s;
   if (k > 0) {
-    AdmitArgs a;
-    a.sal = h->pS[layer];
-    a.K = h->pK[layer];
-    a.V = h->pV[layer];
-    a.bankK = bk;
-    a.bankV = bv;
-    a.cap = h->cap;
-    a.M = h->len[layer];
-    a.N = h->N;
-    a.H = h->heads;
-    a.cand_lo = h->cand_lo;
-    a.k = k;
-    a.idx_out = idx_out;
+    const AdmitArgs a = admit_args(h, layer, h->pK[layer], h->pV[layer], h->pS[layer], k, idx_out);
     RM_CUDA(h, launch_admit(a, h->stream));
     h->prof.launches_admit += 1;
   }
@@ -583,6 +692,8 @@ void regmem_destroy(regmem_t* h) {
   cudaFree(h->part_o);
   cudaFree(h->part_lse);
   cudaFree(h->counters);
+  cudaFree(h->head_done);
+  cudaFree(h->adm_lists);
   if (h->status_host) cudaFreeHost(h->status_host);
   cudaFree(h->stQ);
   cudaFree(h->stOut);

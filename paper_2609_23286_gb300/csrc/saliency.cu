@@ -12,12 +12,21 @@
 // fp32 logits, never on the bf16 P of the attention kernel.
 // The key tile arrives by TMA while every thread gathers its sampled query
 // rows with 16-byte cp.async copies into 128-byte-swizzled tiles; up to four
-// 128-query chunks are resident at once.  Z^T alternates between two
-// 128-column TMEM buffers: the MMA of chunk c+2 is issued as soon as every
-// thread has read chunk c, so it runs under the exponentials of chunk c.
+// 128-query chunks are resident at once, and all of a group's index and LSE
+// loads are issued before any of the copies that depend on them.  Z^T
+// alternates between two 128-column TMEM buffers: the MMA of chunk c+2 is
+// issued as soon as every thread has read chunk c, so it runs under the
+// exponentials of chunk c.
+//
+// Fused admission (Eq. 6): when the launch carries admission arguments, each
+// block sorts its tile's candidates (select.cuh) and stores its best 32, then
+// adds itself to its head's completion counter; the last block of a head
+// merges the tiles' lists into the head's k admitted tokens, appends their K
+// and V rows to the bank and clears the counter for the next launch.
 
 #include "kernels.h"
 #include "ptx.cuh"
+#include "select.cuh"
 
 namespace regmem_dev {
 using namespace ptx;
@@ -36,12 +45,13 @@ constexpr int MAX_CHUNKS = 64;  // sampled queries <= 8192
 
 struct Smem {
   uint8_t k[TILE_BYTES];
-  uint8_t qs[QS][TILE_BYTES];
+  uint8_t qs[QS][TILE_BYTES];  // after the saliency: admission keys and positions
   float lse2[QS][BT];
   uint64_t k_full, mma_bar[2], fin_bar;
   uint32_t tmem_base;
   int abort_flag;
   int never;
+  int last;                    // this block finished its head's saliency last
 };
 // About 83 KB: at most two CTAs share an SM, so their two 256-column TMEM
 // allocations fit the SM's 512 columns.
@@ -56,6 +66,8 @@ struct Params {
   float c;  // scale * log2(e)
   float* sal;
   int* status;
+  int adm_k;       // >= 1: fused admission with these arguments
+  AdmitArgs adm;
 };
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
@@ -65,26 +77,41 @@ __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
-// Gather sampled query rows [chunk*128, chunk*128+128) of head h into a
-// swizzled K-major tile (16-byte chunk c of row r at chunk c ^ (r % 8)), and
-// their LSE (log2 units) into lse2.  Rows past nq are zero with lse2 = +inf,
-// so they contribute exp2(-inf) = 0.
-__device__ __forceinline__ void gather_chunk(const Params& p, int h, int chunk, uint8_t* tile,
-                                             float* lse2, int tid) {
-  const int i = chunk * BT + tid;  // one sampled row per thread
-  const uint32_t base = smem_addr(tile) + tid * 128;
-  if (i < p.nq) {
-    const int tok = p.qidx[i];
-    const uint4* src = reinterpret_cast<const uint4*>(p.Q + ((size_t)tok * p.H + h) * HD);
+// Gather sampled query rows [ch*128, ch*128+128) of head h, chunks g0..g1-1,
+// into swizzled K-major tiles (16-byte chunk c of row r at chunk c ^ (r % 8)),
+// and their LSE (log2 units) into lse2.  Rows past nq are zero with lse2 =
+// +inf, so they contribute exp2(-inf) = 0.  The index loads of all chunks are
+// issued first, then the LSE loads and copies that depend on them.
+__device__ __forceinline__ void gather_group(const Params& p, int h, int g0, int g1, Smem& sm,
+                                             int tid) {
+  int tok[QS];
 #pragma unroll
-    for (int c = 0; c < 8; ++c) cp_async16(base + ((c ^ (tid & 7)) * 16), src + c);
-    lse2[tid] = p.lse[(size_t)h * p.N + tok] * 1.4426950408889634f;
-  } else {
-#pragma unroll
-    for (int c = 0; c < 8; ++c)
-      *reinterpret_cast<uint4*>(tile + tid * 128 + c * 16) = make_uint4(0, 0, 0, 0);
-    lse2[tid] = INFINITY;
+  for (int c = 0; c < QS; ++c) {
+    const int i = (g0 + c) * BT + tid;
+    tok[c] = (g0 + c < g1 && i < p.nq) ? __ldg(p.qidx + i) : -1;
   }
+  float lv[QS];
+#pragma unroll
+  for (int c = 0; c < QS; ++c) lv[c] = tok[c] >= 0 ? p.lse[(size_t)h * p.N + tok[c]] : 0.f;
+#pragma unroll
+  for (int c = 0; c < QS; ++c) {
+    const int ch = g0 + c;
+    if (ch >= g1) break;
+    uint8_t* tile = sm.qs[ch % QS];
+    const uint32_t base = smem_addr(tile) + tid * 128;
+    if (tok[c] >= 0) {
+      const uint4* src = reinterpret_cast<const uint4*>(p.Q + ((size_t)tok[c] * p.H + h) * HD);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) cp_async16(base + ((q ^ (tid & 7)) * 16), src + q);
+    } else {
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        *reinterpret_cast<uint4*>(tile + tid * 128 + q * 16) = make_uint4(0, 0, 0, 0);
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < QS; ++c)
+    if (g0 + c < g1) sm.lse2[(g0 + c) % QS][tid] = tok[c] >= 0 ? lv[c] * 1.4426950408889634f : INFINITY;
 }
 
 __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant__ CUtensorMap tmK,
@@ -138,7 +165,7 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
   for (int g0 = 0; g0 < nchunks && !stop; g0 += QS) {
     const int g1 = min(nchunks, g0 + QS);
     // every MMA that read the chunk buffers has completed (waited below)
-    for (int ch = g0; ch < g1; ++ch) gather_chunk(p, h, ch, sm.qs[ch % QS], sm.lse2[ch % QS], tid);
+    gather_group(p, h, g0, g1, sm, tid);
     cp_async_wait_all();
     fence_proxy_async_smem();
     tc_fence_before();
@@ -193,6 +220,24 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
     tmem_dealloc(tmem, TMEM_COLS);
   }
   if (tid == 0 && sm.abort_flag) atomicOr(p.status, kStatusTimeout);
+  if (p.adm_k < 1) return;
+  // ---- fused admission: this tile's best candidates, then the head's last
+  // block merges the tiles' lists and appends
+  const bool cand = j < p.N && j >= p.adm.cand_lo;
+  uint64_t* lists = reinterpret_cast<uint64_t*>(&sm.qs[0][0]);  // THREADS values
+  sel::block_top_list<THREADS>(cand ? sel::pack_candidate(acc, j) : 0ull, lists,
+                               p.adm.lists + ((size_t)h * nkt + kt) * sel::kListK);
+  __threadfence();  // the list before the count
+  __syncthreads();
+  if (tid == 0) sm.last = atomicAdd(p.adm.done + h, 1) == nkt - 1;
+  __syncthreads();
+  if (!sm.last) return;
+  __threadfence();
+  int* ord = reinterpret_cast<int*>(&sm.qs[1][0]);
+  sel::merge_head_lists<THREADS>(p.adm.lists + (size_t)h * nkt * sel::kListK, nkt, p.adm_k,
+                                 p.adm.cand_lo, lists, ord);
+  sel::append_rows<THREADS>(p.adm, h, ord);
+  if (tid == 0) p.adm.done[h] = 0;  // every block of the head has counted
 }
 
 }  // namespace
@@ -214,6 +259,15 @@ cudaError_t launch_saliency(const SalArgs& a, cudaStream_t s) {
   p.c = a.scale * 1.4426950408889634f;
   p.sal = a.sal;
   p.status = a.status;
+  p.adm_k = 0;
+  if (a.adm) {
+    const int nc = a.N - a.adm->cand_lo;
+    if (a.adm->sal != a.sal || !a.adm->lists || !a.adm->done || nc < 1 || a.adm->k < 1 ||
+        a.adm->k > nc || a.adm->k > sel::kListK)
+      return cudaErrorInvalidValue;
+    p.adm = *a.adm;
+    p.adm_k = a.adm->k;
+  }
   const int nkt = (a.N + BT - 1) / BT;
   saliency_kernel<<<a.H * nkt, THREADS, SMEM_BYTES, s>>>(*a.tmK, p);
   return cudaGetLastError();

@@ -26,6 +26,8 @@ _SIGNATURES = {
     "regmem_attend_frame": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P]),
     "regmem_attend_frame_host": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P]),
     "regmem_admit": (ctypes.c_int, [_P, _I32, _I32, _P]),
+    "regmem_attend_admit": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, _I32, _P]),
+    "regmem_attend_admit_host": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, _I32]),
     "regmem_frame_attention": (ctypes.c_int, [_P, _P, _P, _P, _P]),
     "regmem_reset": (ctypes.c_int, [_P]),
     "regmem_memory_len": (ctypes.c_int, [_P, _I32, ctypes.POINTER(ctypes.c_int64)]),
@@ -156,6 +158,16 @@ def regmem_admit(h, layer, k, idx_out=None):
     return _check(h, load().regmem_admit(h, layer, k, _ptr(idx_out)))
 
 
+def regmem_attend_admit(h, layer, Q, K, V, out, saliency, k, idx_out=None):
+    return _check(h, load().regmem_attend_admit(h, layer, _ptr(Q), _ptr(K), _ptr(V), _ptr(out),
+                                                _ptr(saliency), k, _ptr(idx_out)))
+
+
+def regmem_attend_admit_host(h, layer, Q, K, V, out, saliency, k):
+    return _check(h, load().regmem_attend_admit_host(h, layer, _ptr(Q), _ptr(K), _ptr(V),
+                                                     _ptr(out), _ptr(saliency), k))
+
+
 def regmem_frame_attention(h, Q, K, V, out):
     return _check(h, load().regmem_frame_attention(h, _ptr(Q), _ptr(K), _ptr(V), _ptr(out)))
 
@@ -251,6 +263,12 @@ class RegMem:
 
     def admit(self, layer, k, idx_out=None):
         return regmem_admit(self.h, layer, k, idx_out)
+
+    def attend_admit(self, layer, Q, K, V, out, saliency, k, idx_out=None):
+        return regmem_attend_admit(self.h, layer, Q, K, V, out, saliency, k, idx_out)
+
+    def attend_admit_host(self, layer, Q, K, V, out, saliency, k):
+        return regmem_attend_admit_host(self.h, layer, Q, K, V, out, saliency, k)
 
     def frame_attention(self, Q, K, V, out):
         return regmem_frame_attention(self.h, Q, K, V, out)

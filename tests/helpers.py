@@ -93,6 +93,16 @@ class Stream:
         self.rm.admit(layer, k, idx)
         return idx[:, :k]
 
+    def attend_admit(self, layer, q, k, v, kk):
+        """The one-call step (attention, saliency and admission of kk rows)."""
+        out = torch.empty_like(q)
+        sal = torch.empty(self.H, self.N, dtype=torch.float32, device=q.device)
+        idx = torch.full((self.H, max(kk, 1)), -1, dtype=torch.int32, device="cuda")
+        self.rm.attend_admit(layer, q, k, v, out, sal, kk, idx)
+        lse = torch.empty(self.H, self.N, dtype=torch.float32, device=q.device)
+        self.rm.copy_lse(lse)
+        return out, sal, lse, idx[:, :kk]
+
     def export(self, layer):
         n = self.rm.memory_len(layer)
         bk = torch.empty(self.H, n, 64, dtype=torch.bfloat16)

@@ -15,18 +15,22 @@ from paper_2609_23286_gb300 import regmem
 pytestmark = pytest.mark.gpu
 
 
-def run_stream(L, H, ns, gh, gw, k, frames, seed, ds=2, check_every=1):
+def run_stream(L, H, ns, gh, gw, k, frames, seed, ds=2, check_every=1, fused=False):
     """Free-running stream on GPU and oracle; the oracle adopts the GPU's
     admitted indices after they pass check_indices, so later frames stay
-    comparable.  Returns the number of frames checked."""
+    comparable.  fused: each step is one regmem_attend_admit call (admission
+    inside the saliency kernel) instead of regmem_attend_frame + regmem_admit."""
     st = Stream(L, H, ns, gh, gw, budget=k, max_frames=frames, seed=seed, ds=ds)
     ref = orc.OracleStream(L, H, 64, ns, gh, gw, ds=ds)
     try:
         for t in range(1, frames + 1):
             for layer in range(L):
                 q, kk_, v = st.inputs(layer, t)
-                out, sal, lse = st.attend(layer, q, kk_, v)
-                idx = st.admit(layer, k)
+                if fused:
+                    out, sal, lse, idx = st.attend_admit(layer, q, kk_, v, k)
+                else:
+                    out, sal, lse = st.attend(layer, q, kk_, v)
+                    idx = st.admit(layer, k)
                 torch.cuda.synchronize()
                 r = ref.attend(layer, to64(q), to64(kk_), to64(v))
                 if t % check_every == 0 or t <= 2:
@@ -51,10 +55,11 @@ def run_stream(L, H, ns, gh, gw, k, frames, seed, ds=2, check_every=1):
         st.close()
 
 
-def test_tiny_stream_full_oracle():
+@pytest.mark.parametrize("fused", [False, True])
+def test_tiny_stream_full_oracle(fused):
     """1 layer, 2 heads, 8x8 patches + 5 specials = 69 tokens, 8 frames, k = 1,
     seed 0: the whole stream against the free-running oracle."""
-    run_stream(1, 2, 5, 8, 8, 1, 8, seed=0)
+    run_stream(1, 2, 5, 8, 8, 1, 8, seed=0, fused=fused)
 
 
 def test_vggt_layer_first_frames():
@@ -303,5 +308,126 @@ def test_admit_every_candidate():
         assert (idx.cpu().numpy() == np.arange(ns, ns + nc)[None, :]).all()
         bk, bv = st.export(0)
         assert torch.equal(bk[:, ns + gh * gw + 0:], kk[ns:, :, :].permute(1, 0, 2).cpu())
+    finally:
+        st.close()
+
+
+def test_fused_step_matches_two_calls():
+    """regmem_attend_admit (admission inside the saliency kernel) gives
+    bit-identical outputs, saliency, admitted indices and banks to
+    regmem_attend_frame + regmem_admit on a 1374-token, 16-head stream."""
+    H, ns, gh, gw, k = 16, 5, 37, 37, 14
+    a = Stream(2, H, ns, gh, gw, budget=k, max_frames=6, seed=21)
+    b = Stream(2, H, ns, gh, gw, budget=k, max_frames=6, seed=21)
+    try:
+        for t in range(1, 6):
+            for layer in range(2):
+                q, kk, v = a.inputs(layer, t)
+                o1, s1, l1 = a.attend(layer, q, kk, v)
+                i1 = a.admit(layer, k)
+                o2, s2, l2, i2 = b.attend_admit(layer, q, kk, v, k)
+                torch.cuda.synchronize()
+                assert torch.equal(o1, o2) and torch.equal(s1, s2) and torch.equal(l1, l2)
+                if t > 1:
+                    assert torch.equal(i1, i2)
+        for layer in range(2):
+            assert a.rm.memory_len(layer) == b.rm.memory_len(layer) == ns + gh * gw + 4 * k
+            ka, va = a.export(layer)
+            kb, vb = b.export(layer)
+            assert torch.equal(ka, kb) and torch.equal(va, vb)
+    finally:
+        a.close()
+        b.close()
+
+
+def test_fused_uniform_keys_and_every_candidate():
+    """The fused selection: uniform saliency ties to the lowest indices, and
+    k = all candidates admits every patch token in order."""
+    H, ns, gh, gw = 4, 5, 8, 8
+    nc = gh * gw
+    for k, zero_keys in ((20, True), (nc, False)):
+        st = Stream(1, H, ns, gh, gw, budget=k, max_frames=3, seed=22)
+        try:
+            for t in (1, 2):
+                q, kk, v = st.inputs(0, t)
+                if zero_keys:
+                    kk = torch.zeros_like(kk)
+                out, sal, lse, idx = st.attend_admit(0, q, kk, v, k)
+            torch.cuda.synchronize()
+            assert (idx.cpu().numpy() == np.arange(ns, ns + k)[None, :]).all()
+            bk, _ = st.export(0)
+            assert torch.equal(bk[:, ns + gh * gw:], kk[ns:ns + k].permute(1, 0, 2).cpu())
+        finally:
+            st.close()
+
+
+def test_fused_host_entry_point_and_errors():
+    H, ns, gh, gw, k = 16, 5, 37, 37, 14
+    N = ns + gh * gw
+    a = Stream(1, H, ns, gh, gw, budget=k, max_frames=4, seed=23)
+    b = Stream(1, H, ns, gh, gw, budget=k, max_frames=4, seed=23)
+    try:
+        for t in range(1, 4):
+            q, kk, v = a.inputs(0, t)
+            o_d, s_d, _, _ = a.attend_admit(0, q, kk, v, k)
+            hq, hk, hv = q.cpu().pin_memory(), kk.cpu().pin_memory(), v.cpu().pin_memory()
+            ho = torch.empty_like(hq).pin_memory()
+            hs = torch.empty(H, N, dtype=torch.float32).pin_memory()
+            b.rm.attend_admit_host(0, hq, hk, hv, ho, hs, k)
+            b.rm.synchronize()
+            torch.cuda.synchronize()
+            assert torch.equal(ho, o_d.cpu()) and torch.equal(hs, s_d.cpu())
+        assert a.rm.memory_len(0) == b.rm.memory_len(0) == N + 2 * k
+        q, kk, v = a.inputs(0, 4)
+        out = torch.empty_like(q)
+        sal = torch.empty(H, N, device="cuda")
+        with pytest.raises(regmem.RegmemError) as e:
+            a.rm.attend_admit(0, q, kk, v, out, sal, k + 1)
+        assert e.value.status == regmem.ERR_ARG               # k above the budget
+        a.rm.attend_frame(0, q, kk, v, out, sal)
+        with pytest.raises(regmem.RegmemError) as e:
+            a.rm.attend_admit(0, q, kk, v, out, sal, k)
+        assert e.value.status == regmem.ERR_STATE             # attend pending
+        a.rm.admit(0, 0)
+        assert a.rm.memory_len(0) == N + 2 * k                # nothing appended by the refusals
+        a.rm.synchronize()
+    finally:
+        a.close()
+        b.close()
+
+
+@pytest.mark.parametrize("pattern", ["duplicates", "constant", "spread"])
+@pytest.mark.parametrize("k", [14, 32, 33])
+def test_selection_on_crafted_saliency(pattern, k):
+    """The admission selection against the oracle's sort on crafted saliency
+    written between attend and admit (the library reads the caller's saliency
+    buffer at admit time): many exact ties, a constant row, and a wide value
+    range across 1369 candidates; k = 14 and 32 take the distributed list
+    selection, k = 33 the single-block radix selection."""
+    H, ns, gh, gw = 16, 5, 37, 37
+    N = ns + gh * gw
+    st = Stream(1, H, ns, gh, gw, budget=k, max_frames=3, seed=24)
+    g = torch.Generator().manual_seed(25)
+    try:
+        q, kk, v = st.inputs(0, 1)
+        st.attend(0, q, kk, v)
+        st.admit(0, k)
+        q, kk, v = st.inputs(0, 2)
+        out = torch.empty_like(q)
+        sal = torch.empty(H, N, device="cuda")
+        st.rm.attend_frame(0, q, kk, v, out, sal)
+        if pattern == "duplicates":
+            crafted = torch.randint(0, 6, (H, N), generator=g).float() * 0.25
+        elif pattern == "constant":
+            crafted = torch.full((H, N), 3.5)
+        else:
+            crafted = torch.exp(torch.randn(H, N, generator=g) * 8.0)
+        sal.copy_(crafted.to("cuda"))
+        idx = torch.full((H, k), -1, dtype=torch.int32, device="cuda")
+        st.rm.admit(0, k, idx)
+        torch.cuda.synchronize()
+        c = crafted.double().numpy()
+        for h in range(H):
+            assert list(idx[h].cpu().numpy()) == orc.topk_admission(c[h], ns, k), f"head {h}"
     finally:
         st.close()
