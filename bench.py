@@ -71,6 +71,13 @@ ATTN_TRAFFIC_NOTE = ("ncu dram bytes of the frame-1001 launch (mean attended len
                      "layer's bank)")
 
 
+# Attention launches bracketed by CUDA events inside the timed region: every
+# 8th.  Kernels are launched to overlap their predecessor's tail; an event
+# pair removes that overlap at its two boundaries, so a sparse sample keeps
+# the timed step close to an unobserved one.
+PROFILE_EVERY = 8
+
+
 def describe(cfg, name):
     N = cfg["ns"] + cfg["gh"] * cfg["gw"]
     s = (f"{name}: {cfg['layers']} layers x {cfg['heads']} heads x 64, {N} tok/frame "
@@ -367,7 +374,7 @@ def gpu_arm(args, cfg, cfg_name):
 
     clocks = ClockSampler(local_rank)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    rm.profile_enable(1)
+    rm.profile_enable(PROFILE_EVERY)
     barrier()
     torch.cuda.synchronize()
     clocks.start()
@@ -471,12 +478,15 @@ def gpu_arm(args, cfg, cfg_name):
             "traffic": ATTN_TRAFFIC_BYTES_PER_LAUNCH,
             "traffic_note": ATTN_TRAFFIC_NOTE if ATTN_TRAFFIC_BYTES_PER_LAUNCH else None,
             "launches": prof.attention_timed,
+            "launches_sampled_every": PROFILE_EVERY,
+            "launches_total": prof.launches_attention,
             "ctas": prof.attention_ctas,
             "ctas_per_sm": prof.attention_ctas_per_sm,
             "mean_launch_ms": round(attn_ms_mean, 5),
             "algorithmic_flops_per_launch": prof.attention_flops / max(prof.attention_timed, 1),
             "algorithmic_bytes_per_launch": prof.attention_bytes / max(prof.attention_timed, 1),
-            "share_of_step": round(prof.attention_ms / ms_local, 4) if ms_local else None,
+            "share_of_step": (round(attn_ms_mean * prof.launches_attention / ms_local, 4)
+                              if ms_local else None),
         },
         "gpu_launches": launches,
         "clocks": clk,

@@ -131,9 +131,11 @@ REGMEM_API regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int
 
 /* regmem_attend_frame followed by regmem_admit(layer, k, idx_out), in one
  * call: the whole per-frame step of one layer (Eq. 3, the LSE-Saliency of
- * Sec. 3.3, then Eq. 4 or Eq. 6).  The admission runs inside the saliency
- * kernel (the last block of each head selects and appends), so it needs no
- * launch of its own.  Arguments, layouts, k range and errors as in the two
+ * Sec. 3.3, then Eq. 4 or Eq. 6).  For k <= 32 the admission runs inside the
+ * saliency kernel (each key tile keeps its best candidates, the last block of
+ * each head merges them and appends), so it needs no launch of its own;
+ * larger k takes a separate selection kernel.  Arguments, layouts, k range
+ * and errors as in the two
  * calls; every check (including k and capacity) is made before anything is
  * enqueued.  The library keeps no pointer after the call: K, V and saliency
  * need only stay valid until the enqueued work has run.
@@ -227,9 +229,9 @@ REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_frame_desc* fd
 /* Launch counters and kernel timing, for measurement tools.
  * Counters cover every kernel this handle launched since the last
  * regmem_profile_enable.  When time_attention is set, CUDA events are
- * recorded on the handle's stream immediately before and after each launch
- * of the attention kernel (one event pair per attend), and attention_ms is
- * the sum of those event intervals; the other kernels are not bracketed. */
+ * recorded on the handle's stream immediately before and after the sampled
+ * launches of the attention kernel, and attention_ms is the sum of those
+ * event intervals; the other kernels are not bracketed. */
 typedef struct regmem_profile {
   int64_t launches_attention; /* attention kernel (attend and frame attention)  */
   int64_t launches_saliency;  /* LSE-saliency kernel                            */
@@ -244,8 +246,11 @@ typedef struct regmem_profile {
   int32_t attention_ctas_per_sm; /* resident attention CTAs per SM (occupancy) */
 } regmem_profile;
 
-/* Resets the counters; time_attention = 1 also brackets attention launches
- * with events (time_attention = 0 stops it). */
+/* Resets the counters; time_attention = n >= 1 also brackets every n-th
+ * attention launch with events (0 stops it).  Kernels are launched so that
+ * each may start while its predecessor in the stream finishes; an event pair
+ * between two launches removes that overlap at those two boundaries, so a
+ * sparse sample (n of 8 or more) perturbs a long run least. */
 REGMEM_API regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention);
 
 /* Waits for the handle's stream and fills *out. */

@@ -13,9 +13,12 @@
 // the bank's first N rows.
 
 #include "kernels.h"
+#include "ptx.cuh"
 #include "select.cuh"
 
 namespace regmem_dev {
+using ptx::grid_dep_wait;
+using ptx::grid_dep_launch;
 
 namespace {
 
@@ -26,6 +29,8 @@ constexpr int HD = kHeadDim;
 __global__ void __launch_bounds__(THREADS) admit_kernel(AdmitArgs a) {
   __shared__ int red[sel::red_words<THREADS>()], ws[WARPS], bc[2];
   extern __shared__ uint32_t dyn[];  // keys [n], then the admitted positions [k]
+  grid_dep_wait();  // the saliency kernel has finished
+  grid_dep_launch();
   const int h = blockIdx.x;
   const int n = a.N - a.cand_lo;
   uint32_t* keys = dyn;
@@ -41,6 +46,8 @@ __global__ void __launch_bounds__(LT) admit_lists_kernel(AdmitArgs a, int nkt) {
   __shared__ uint64_t lists[LT];
   __shared__ int ord[sel::kListK];
   __shared__ int last;
+  grid_dep_wait();  // the saliency kernel has finished
+  grid_dep_launch();
   const int h = blockIdx.x / nkt, kt = blockIdx.x - h * nkt, tid = threadIdx.x;
   const int j = kt * LT + tid;
   const bool cand = j < a.N && j >= a.cand_lo;
@@ -60,6 +67,8 @@ __global__ void __launch_bounds__(LT) admit_lists_kernel(AdmitArgs a, int nkt) {
 
 __global__ void anchor_kernel(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
                               __nv_bfloat16* bankV, long long cap, int N, int H) {
+  grid_dep_wait();
+  grid_dep_launch();
   const long long total = (long long)N * H * 8;  // 16-byte chunks per tensor
   for (long long w = blockIdx.x * (long long)blockDim.x + threadIdx.x; w < 2 * total;
        w += (long long)gridDim.x * blockDim.x) {
@@ -88,11 +97,9 @@ cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s) {
   if (a.k == 0) return cudaSuccess;
   if (a.k <= sel::kListK && a.lists && a.done) {
     const int nkt = (a.N + LT - 1) / LT;
-    admit_lists_kernel<<<a.H * nkt, LT, 0, s>>>(a, nkt);
-  } else {
-    admit_kernel<<<a.H, THREADS, (size_t)(nc + a.k) * sizeof(int), s>>>(a);
+    return launch_pdl(admit_lists_kernel, dim3(a.H * nkt), dim3(LT), 0, s, a, nkt);
   }
-  return cudaGetLastError();
+  return launch_pdl(admit_kernel, dim3(a.H), dim3(THREADS), (size_t)(nc + a.k) * sizeof(int), s, a);
 }
 
 cudaError_t launch_anchor(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
@@ -100,8 +107,7 @@ cudaError_t launch_anchor(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_b
   const long long work = 2LL * N * H * 8;
   int blocks = (int)((work + 255) / 256);
   if (blocks > 4096) blocks = 4096;
-  anchor_kernel<<<blocks, 256, 0, s>>>(K, V, bankK, bankV, cap, N, H);
-  return cudaGetLastError();
+  return launch_pdl(anchor_kernel, dim3(blocks), dim3(256), 0, s, K, V, bankK, bankV, cap, N, H);
 }
 
 }  // namespace regmem_dev

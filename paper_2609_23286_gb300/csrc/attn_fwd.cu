@@ -21,8 +21,12 @@
 // merging piece waits (bounded) for the count with acquire loads and folds
 // the partials into its own result,
 //     LSE = log sum_p exp(LSE_p),  O = sum_p exp(LSE_p - LSE) O_p,
-// then resets the counter.  CTAs wait on one another, so the kernel is
-// launched cooperatively (all CTAs resident, one per SM).
+// then resets the counter.  The grid is one CTA per SM, so every CTA becomes
+// resident once the kernels launched before it have left the SMs; the wait is
+// bounded all the same, and on expiry the status word reports it.
+// The kernel may start while its predecessor in the stream finishes: barrier
+// setup and the TMEM allocation run before griddepcontrol.wait, everything
+// that reads inputs or writes outputs after it.
 //
 // CTA layout, warp-specialised (12 warps, three warpgroups):
 //   warp 0       TMA producer: both Q tiles of a unit, then K and V tiles
@@ -193,6 +197,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
+  grid_dep_wait();    // the previous kernel's writes are visible, its reads done
+  grid_dep_launch();  // the next kernel may be scheduled as SMs free up
 
   if (warp < 4) {
    setmaxnreg_dec<REGS_CTRL>();
@@ -616,19 +622,8 @@ cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_b
   if (a.grid < 1 || (long long)a.grid > p.total) return cudaErrorInvalidValue;
   cudaError_t e;
   if (ev_before && (e = cudaEventRecord(ev_before, s)) != cudaSuccess) return e;
-  // Cooperative: the merging pieces wait for pieces of other CTAs, so every
-  // CTA must be resident (the launch fails rather than oversubscribe).
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.grid);
-  cfg.blockDim = dim3(THREADS);
-  cfg.dynamicSmemBytes = SMEM_BYTES;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;
-  attr[0].val.cooperative = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, attn_fwd_kernel, *a.tmQ, *a.tmK, *a.tmV, *a.tmBK, *a.tmBV, p);
+  e = launch_pdl(attn_fwd_kernel, dim3(a.grid), dim3(THREADS), SMEM_BYTES, s, *a.tmQ, *a.tmK, *a.tmV,
+                 *a.tmBK, *a.tmBV, p);
   if (e != cudaSuccess) return e;
   if (ev_after && (e = cudaEventRecord(ev_after, s)) != cudaSuccess) return e;
   return cudaSuccess;

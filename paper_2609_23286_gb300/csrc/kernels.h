@@ -9,6 +9,25 @@
 
 namespace regmem_dev {
 
+// Launches `kernel` with programmatic stream serialization: it may start
+// while the previous kernel in the stream finishes, and waits for it inside
+// (griddepcontrol.wait) before touching what that kernel may read or write.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 constexpr int kHeadDim = 64;    // channels per head handled by the kernels
 constexpr int kTile = 128;      // query rows / key rows per tile
 

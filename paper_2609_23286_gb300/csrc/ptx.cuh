@@ -355,6 +355,17 @@ __device__ __forceinline__ void tmem_wait_ld128(uint32_t (&r)[128]) {
                : "memory");
 }
 
+// Programmatic dependent launch.  grid_dep_wait() returns once every grid
+// this one depends on has completed and its memory is visible (immediately
+// when the launch had no such dependency); grid_dep_launch() lets the grids
+// that depend on this one be scheduled before it finishes.  Every kernel
+// calls grid_dep_launch() only after its own grid_dep_wait(), so a grid that
+// starts early can rely on everything before its predecessor being complete.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // bar.red.or over a named barrier: every participating thread gets the OR of
 // the predicates, so a decision taken on it is uniform across the group.
 __device__ __forceinline__ int named_bar_red_or(int id, int nthreads, int pred) {

@@ -58,7 +58,8 @@ struct regmem {
 
   // measurement (regmem_profile_*)
   regmem_profile prof = {};
-  bool time_attention = false;
+  int time_every = 0;          // time every n-th attention launch (0: none)
+  long long attn_launch_no = 0;
   std::vector<cudaEvent_t> ev_ring;  // pairs: [2i] before, [2i+1] after
   std::vector<int> ev_busy;
   size_t ev_next = 0;
@@ -196,7 +197,9 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   const long long G = pl.total < h->attn_grid ? pl.total : h->attn_grid;
   a.grid = (int)G;
   cudaEvent_t eb = nullptr, ea = nullptr;
-  if (h->time_attention) {
+  const bool timed = h->time_every > 0 && h->attn_launch_no % h->time_every == 0;
+  ++h->attn_launch_no;
+  if (timed) {
     if (h->ev_ring.empty()) {
       h->ev_ring.resize(2 * kEventPairs);
       h->ev_busy.assign(kEventPairs, 0);
@@ -214,7 +217,7 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   h->prof.attention_ctas_per_sm = h->attn_ctas_per_sm;
   const double L = (double)M + h->N;
   h->prof.launches_attention += 1;
-  if (h->time_attention) {
+  if (timed) {
     h->prof.attention_timed += 1;
     h->prof.attention_flops += 4.0 * h->N * L * kHeadDim * h->heads;
     h->prof.attention_bytes += (2.0 * h->N * h->heads * kHeadDim * 2)   // Q in, O out
@@ -662,7 +665,8 @@ regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention) {
       if (h->ev_busy[i]) RM_CUDA(h, harvest_pair(h, i));
   }
   h->prof = regmem_profile{};
-  h->time_attention = time_attention != 0;
+  h->time_every = time_attention > 0 ? time_attention : 0;
+  h->attn_launch_no = 0;
   return REGMEM_OK;
 }
 

@@ -78,21 +78,16 @@ __device__ __forceinline__ void cp_async_wait_all() {
 }
 
 // Gather sampled query rows [ch*128, ch*128+128) of head h, chunks g0..g1-1,
-// into swizzled K-major tiles (16-byte chunk c of row r at chunk c ^ (r % 8)),
-// and their LSE (log2 units) into lse2.  Rows past nq are zero with lse2 =
-// +inf, so they contribute exp2(-inf) = 0.  The index loads of all chunks are
-// issued first, then the LSE loads and copies that depend on them.
-__device__ __forceinline__ void gather_group(const Params& p, int h, int g0, int g1, Smem& sm,
-                                             int tid) {
-  int tok[QS];
+// into swizzled K-major tiles (16-byte chunk c of row r at chunk c ^ (r % 8)).
+// The index loads of all chunks are issued first, then the copies that
+// depend on them; tok[c] keeps each thread's row (-1 past nq: a zero row).
+__device__ __forceinline__ void gather_rows(const Params& p, int h, int g0, int g1, Smem& sm, int tid,
+                                            int (&tok)[QS]) {
 #pragma unroll
   for (int c = 0; c < QS; ++c) {
     const int i = (g0 + c) * BT + tid;
     tok[c] = (g0 + c < g1 && i < p.nq) ? __ldg(p.qidx + i) : -1;
   }
-  float lv[QS];
-#pragma unroll
-  for (int c = 0; c < QS; ++c) lv[c] = tok[c] >= 0 ? p.lse[(size_t)h * p.N + tok[c]] : 0.f;
 #pragma unroll
   for (int c = 0; c < QS; ++c) {
     const int ch = g0 + c;
@@ -109,6 +104,15 @@ __device__ __forceinline__ void gather_group(const Params& p, int h, int g0, int
         *reinterpret_cast<uint4*>(tile + tid * 128 + q * 16) = make_uint4(0, 0, 0, 0);
     }
   }
+}
+
+// The LSE of the gathered rows, in log2 units, into lse2 (+inf for zero rows,
+// so they contribute exp2(-inf) = 0).
+__device__ __forceinline__ void gather_lse(const Params& p, int h, int g0, int g1, Smem& sm, int tid,
+                                           const int (&tok)[QS]) {
+  float lv[QS];
+#pragma unroll
+  for (int c = 0; c < QS; ++c) lv[c] = tok[c] >= 0 ? p.lse[(size_t)h * p.N + tok[c]] : 0.f;
 #pragma unroll
   for (int c = 0; c < QS; ++c)
     if (g0 + c < g1) sm.lse2[(g0 + c) % QS][tid] = tok[c] >= 0 ? lv[c] * 1.4426950408889634f : INFINITY;
@@ -162,10 +166,18 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
     mma_commit(b_mma[ch & 1]);
   };
   bool stop = false;
+  // The key tile (issued above) and the sampled rows come from the frame's
+  // inputs, which precede the attention kernel: they are loaded while that
+  // kernel finishes.  The LSE it writes is read after the wait.
+  int tok[QS];
+  gather_rows(p, h, 0, min(nchunks, QS), sm, tid, tok);
+  grid_dep_wait();
+  grid_dep_launch();
   for (int g0 = 0; g0 < nchunks && !stop; g0 += QS) {
     const int g1 = min(nchunks, g0 + QS);
     // every MMA that read the chunk buffers has completed (waited below)
-    gather_group(p, h, g0, g1, sm, tid);
+    if (g0 > 0) gather_rows(p, h, g0, g1, sm, tid, tok);
+    gather_lse(p, h, g0, g1, sm, tid, tok);
     cp_async_wait_all();
     fence_proxy_async_smem();
     tc_fence_before();
@@ -269,8 +281,7 @@ cudaError_t launch_saliency(const SalArgs& a, cudaStream_t s) {
     p.adm_k = a.adm->k;
   }
   const int nkt = (a.N + BT - 1) / BT;
-  saliency_kernel<<<a.H * nkt, THREADS, SMEM_BYTES, s>>>(*a.tmK, p);
-  return cudaGetLastError();
+  return launch_pdl(saliency_kernel, dim3(a.H * nkt), dim3(THREADS), SMEM_BYTES, s, *a.tmK, p);
 }
 
 }  // namespace regmem_dev
