@@ -208,7 +208,7 @@ REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
  * All pointers 16-byte aligned (status 4-byte aligned).
  *
  * Scratch: the kernels' split partials, LSE rows and sampled-query list live
- * in one file-scope device array of 11.8 MB that every GPU which loads this
+ * in one file-scope device array of 22.3 MB that every GPU which loads this
  * library holds until the process exits.  Limits, rejected with
  * REGMEM_ERR_UNSUPPORTED before anything is enqueued: heads * N <= 262144,
  * N <= 65536, sampled queries <= 8192, and the attention grid (one CTA per
@@ -237,8 +237,10 @@ typedef struct regmem_profile {
   int64_t launches_saliency;  /* LSE-saliency kernel                            */
   int64_t launches_admit;     /* top-k + append kernel                          */
   int64_t launches_anchor;    /* first-frame copy kernel                        */
+  int64_t launches_combine;   /* merge of units split between attention CTAs   */
   int64_t attention_timed;    /* attention launches with an event pair          */
-  double attention_ms;        /* summed event time of those launches            */
+  double attention_ms;        /* summed event time of those launches (attention
+                                 kernel plus the merge of split units)          */
   double attention_flops;     /* algorithmic 4*N*(M+N)*64*H of those launches   */
   double attention_bytes;     /* algorithmic HBM bytes of those launches:
                                  Q, O, K/V of the attended rows, LSE           */

@@ -13,17 +13,12 @@
 // consecutive 128-row query tiles); the (unit, key tile) space is cut into
 // `grid` contiguous equal ranges, one per CTA (one CTA per SM).  A unit whose
 // key tiles all fall in one CTA is finished there (O in bf16 and LSE written
-// directly).  For a unit cut between CTAs, the piece holding its first key
-// tile merges (it is the last piece of its CTA's range, processed after the
-// unit's other pieces, which are the first pieces of the following CTAs):
-// each other piece stores its normalised fp32 partial (O_p, LSE_p) and
-// increments a per-(unit, query tile) counter with release semantics; the
-// merging piece waits (bounded) for the count with acquire loads and folds
-// the partials into its own result,
-//     LSE = log sum_p exp(LSE_p),  O = sum_p exp(LSE_p - LSE) O_p,
-// then resets the counter.  The grid is one CTA per SM, so every CTA becomes
-// resident once the kernels launched before it have left the SMs; the wait is
-// bounded all the same, and on expiry the status word reports it.
+// directly).  A unit cut between CTAs leaves one normalised fp32 partial
+// (O_p, LSE_p) per piece, in a slot of the CTA that computed it (its first or
+// its last piece), and attn_combine_kernel, launched right behind, folds
+// each split unit's pieces in CTA order,
+//     LSE = log sum_p exp(LSE_p),  O = sum_p exp(LSE_p - LSE) O_p.
+// No CTA waits for another.
 // The kernel may start while its predecessor in the stream finishes: barrier
 // setup and the TMEM allocation run before griddepcontrol.wait, everything
 // that reads inputs or writes outputs after it.
@@ -113,9 +108,8 @@ struct Params {
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  float* part_o;    // [grid][256][64]: the first piece of each CTA, when it is a non-merging piece
-  float* part_lse;  // [grid][256]
-  int* counters;    // [units][2], zero between launches
+  float* part_o;    // [grid][2][256][64]: partials of each CTA's first / last piece
+  float* part_lse;  // [grid][2][256]
   int* status;
 };
 
@@ -197,8 +191,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  grid_dep_wait();    // the previous kernel's writes are visible, its reads done
-  grid_dep_launch();  // the next kernel may be scheduled as SMs free up
+  grid_dep_wait();  // the previous kernel's writes are visible, its reads done
 
   if (warp < 4) {
    setmaxnreg_dec<REGS_CTRL>();
@@ -477,85 +470,18 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           p.lse[(size_t)pc.h * p.N + q] = lse_val;
         }
-      } else if (pc.j0 > 0) {
-        // a later piece of a split unit: hand the partial to the merging piece
-        const size_t pr = (size_t)b * UROWS + t * BM + row;
+      } else {
+        // a piece of a unit split between CTAs: its normalised partial goes
+        // to the CTA's slot (0: the CTA's first piece, 1: its last piece);
+        // attn_combine_kernel merges the unit's pieces
+        const int which = (x - n == x_begin) ? 0 : 1;
+        const size_t pr = ((size_t)b * 2 + which) * UROWS + t * BM + row;
         float4* dst = reinterpret_cast<float4*>(p.part_o + pr * HD);
 #pragma unroll
         for (int c4 = 0; c4 < 16; ++c4)
           dst[c4] = make_float4(__uint_as_float(orr[c4 * 4 + 0]) * inv_l, __uint_as_float(orr[c4 * 4 + 1]) * inv_l,
                                 __uint_as_float(orr[c4 * 4 + 2]) * inv_l, __uint_as_float(orr[c4 * 4 + 3]) * inv_l);
         p.part_lse[pr] = lse_val;
-        named_bar_sync(1 + t, BM);
-        if ((warp & 3) == 3 && lane == 0) red_release_add(&p.counters[pc.u * 2 + t], 1);
-      } else {
-        // first piece of a split unit: wait for the other pieces and merge
-        const long long T = p.total;
-        const int b_hi = cta_of((long long)pc.u * p.nkv + p.nkv - 1, G, T);
-        const int others = b_hi - b;  // pieces in CTAs b+1 .. b_hi
-        const bool leader = (warp & 3) == 3 && lane == 0;
-        if (leader) {
-          int* cnt = &p.counters[pc.u * 2 + t];
-          bool done = ld_acquire(cnt) >= others;
-          const uint64_t t0 = done ? 0 : globaltimer_ns();
-          while (!done) {
-            if (*abort_flag || globaltimer_ns() - t0 > WAIT_NS) {
-              *abort_flag = 1;
-              break;
-            }
-            __nanosleep(64);
-            done = ld_acquire(cnt) >= others;
-          }
-          *cnt = 0;  // every other piece has counted: ready for the next launch
-        }
-        named_bar_sync(1 + t, BM);
-        if (*abort_flag) {
-          stop = true;
-        } else {
-          // online merge: own result first, then the partials in CTA order
-          float m = lse_val, den = 1.f;
-          float acc[HD];
-#pragma unroll
-          for (int i = 0; i < HD; ++i) acc[i] = __uint_as_float(orr[i]) * inv_l;
-          for (int bb = b + 1; bb <= b_hi; ++bb) {
-            const size_t pr = (size_t)bb * UROWS + t * BM + row;
-            const float lp = __ldcg(p.part_lse + pr);
-            const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD);
-            const float mn = fmaxf(m, lp);
-            const float a_old = ex2((m - mn) * 1.4426950408889634f);
-            const float a_new = ex2((lp - mn) * 1.4426950408889634f);
-            den = den * a_old + a_new;
-#pragma unroll
-            for (int g = 0; g < 4; ++g) {  // 16 columns at a time
-              float4 v[4];
-#pragma unroll
-              for (int c4 = 0; c4 < 4; ++c4) v[c4] = __ldcg(src + g * 4 + c4);
-#pragma unroll
-              for (int c4 = 0; c4 < 4; ++c4) {
-                const int e = (g * 4 + c4) * 4;
-                acc[e + 0] = acc[e + 0] * a_old + v[c4].x * a_new;
-                acc[e + 1] = acc[e + 1] * a_old + v[c4].y * a_new;
-                acc[e + 2] = acc[e + 2] * a_old + v[c4].z * a_new;
-                acc[e + 3] = acc[e + 3] * a_old + v[c4].w * a_new;
-              }
-            }
-            m = mn;
-          }
-          const float inv = 1.f / den;
-          if (q < p.N) {
-            uint4* o = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + pc.h) * HD);
-#pragma unroll
-            for (int c8 = 0; c8 < 8; ++c8) {
-              uint4 w4;
-              w4.x = pack_bf16x2(acc[c8 * 8 + 0] * inv, acc[c8 * 8 + 1] * inv);
-              w4.y = pack_bf16x2(acc[c8 * 8 + 2] * inv, acc[c8 * 8 + 3] * inv);
-              w4.z = pack_bf16x2(acc[c8 * 8 + 4] * inv, acc[c8 * 8 + 5] * inv);
-              w4.w = pack_bf16x2(acc[c8 * 8 + 6] * inv, acc[c8 * 8 + 7] * inv);
-              o[c8] = w4;
-            }
-            p.lse[(size_t)pc.h * p.N + q] = m + __logf(den);
-          }
-        }
       }
     }
   }
@@ -566,6 +492,103 @@ __global__ void __launch_bounds__(THREADS, 1)
     tmem_dealloc(tmem, TMEM_COLS);
   }
   if (tid == 0 && sm.abort_flag) atomicOr(p.status, kStatusTimeout);
+  // The merge kernel behind is released only as CTAs finish: released at the
+  // start, its small blocks took SMs as they freed up and held them while
+  // waiting, which measured 25 us slower per launch.
+  grid_dep_launch();
+}
+
+// Merges the pieces of every split unit: one block per (unit, query tile),
+// four threads per query row (16 of its 64 channels each, so the partial
+// rows are read coalesced), and the loads of up to CMB_MAXP pieces issued
+// together so the merge costs one memory round trip.  Blocks of units
+// finished in one CTA, and second tiles of units that have none, return at
+// once.  Pieces are folded in CTA order, so the result does not depend on
+// which CTA finished first.
+constexpr int CMB_THREADS = 4 * BM;
+constexpr int CMB_MAXP = 4;
+
+__global__ void __launch_bounds__(CMB_THREADS) attn_combine_kernel(const Params p, int G) {
+  __shared__ long long s_slot[64];  // row-0 partial index of each piece, in CTA order
+  __shared__ int s_np;
+  grid_dep_wait();  // every piece's partial is stored
+  grid_dep_launch();
+  const int u = blockIdx.x >> 1, t = blockIdx.x & 1;
+  const int h = u / p.nqp, qp = u - h * p.nqp;
+  if (t == 1 && 2 * qp + 1 >= p.nqt) return;
+  const long long T = p.total;
+  const long long x0 = (long long)u * p.nkv;
+  if (threadIdx.x == 0) {
+    const int b_lo = cta_of(x0, G, T), b_hi = cta_of(x0 + p.nkv - 1, G, T);
+    int np = 0;
+    if (b_hi > b_lo) {
+      for (int bb = b_lo; bb <= b_hi && np < 64; ++bb) {
+        const int which = range_begin(bb, G, T) >= x0 ? 0 : 1;
+        s_slot[np++] = ((long long)bb * 2 + which) * UROWS + t * BM;
+      }
+    }
+    s_np = np;
+  }
+  __syncthreads();
+  const int np = s_np;
+  if (np == 0) return;  // finished in one CTA
+  const int row = threadIdx.x >> 2, qtr = threadIdx.x & 3;
+  const int q = (2 * qp + t) * BM + row;
+  float lp[CMB_MAXP];
+  float4 v[CMB_MAXP][4];
+#pragma unroll
+  for (int i = 0; i < CMB_MAXP; ++i) {
+    if (i < np) {
+      const size_t pr = (size_t)s_slot[i] + row;
+      lp[i] = __ldcg(p.part_lse + pr);
+      const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD) + qtr * 4;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) v[i][c] = __ldcg(src + c);
+    }
+  }
+  float m = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < CMB_MAXP; ++i)
+    if (i < np) m = fmaxf(m, lp[i]);
+  for (int i = CMB_MAXP; i < np; ++i) m = fmaxf(m, __ldcg(p.part_lse + (size_t)s_slot[i] + row));
+  float den = 0.f, acc[16];
+#pragma unroll
+  for (int c = 0; c < 16; ++c) acc[c] = 0.f;
+  auto fold = [&](float l, const float4 (&w)[4]) {
+    const float a = ex2((l - m) * 1.4426950408889634f);
+    den += a;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      acc[c * 4 + 0] += w[c].x * a;
+      acc[c * 4 + 1] += w[c].y * a;
+      acc[c * 4 + 2] += w[c].z * a;
+      acc[c * 4 + 3] += w[c].w * a;
+    }
+  };
+#pragma unroll
+  for (int i = 0; i < CMB_MAXP; ++i)
+    if (i < np) fold(lp[i], v[i]);
+  for (int i = CMB_MAXP; i < np; ++i) {  // units cut into more pieces than are prefetched
+    const size_t pr = (size_t)s_slot[i] + row;
+    const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD) + qtr * 4;
+    float4 w[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) w[c] = __ldcg(src + c);
+    fold(__ldcg(p.part_lse + pr), w);
+  }
+  if (q >= p.N) return;
+  const float inv = 1.f / den;
+  uint4* o = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + h) * HD) + qtr * 2;
+#pragma unroll
+  for (int c8 = 0; c8 < 2; ++c8) {
+    uint4 w4;
+    w4.x = pack_bf16x2(acc[c8 * 8 + 0] * inv, acc[c8 * 8 + 1] * inv);
+    w4.y = pack_bf16x2(acc[c8 * 8 + 2] * inv, acc[c8 * 8 + 3] * inv);
+    w4.z = pack_bf16x2(acc[c8 * 8 + 4] * inv, acc[c8 * 8 + 5] * inv);
+    w4.w = pack_bf16x2(acc[c8 * 8 + 6] * inv, acc[c8 * 8 + 7] * inv);
+    o[c8] = w4;
+  }
+  if (qtr == 0) p.lse[(size_t)h * p.N + q] = m + __logf(den);
 }
 
 Params make_params(const AttnArgs& a) {
@@ -584,7 +607,6 @@ Params make_params(const AttnArgs& a) {
   p.lse = a.lse;
   p.part_o = a.part_o;
   p.part_lse = a.part_lse;
-  p.counters = a.counters;
   p.status = a.status;
   return p;
 }
@@ -624,6 +646,9 @@ cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_b
   if (ev_before && (e = cudaEventRecord(ev_before, s)) != cudaSuccess) return e;
   e = launch_pdl(attn_fwd_kernel, dim3(a.grid), dim3(THREADS), SMEM_BYTES, s, *a.tmQ, *a.tmK, *a.tmV,
                  *a.tmBK, *a.tmBV, p);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(attn_combine_kernel, dim3((unsigned)(p.total / p.nkv) * 2), dim3(CMB_THREADS), 0, s, p,
+                 a.grid);
   if (e != cudaSuccess) return e;
   if (ev_after && (e = cudaEventRecord(ev_after, s)) != cudaSuccess) return e;
   return cudaSuccess;

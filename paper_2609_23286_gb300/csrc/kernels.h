@@ -46,9 +46,8 @@ struct AttnArgs {
   float scale;
   __nv_bfloat16* out;       // [N][H][64]
   float* lse;               // [H][N]
-  float* part_o;            // [grid][kUnitRows][64] split-piece partial outputs
-  float* part_lse;          // [grid][kUnitRows]
-  int* counters;            // [units][2] piece counters, all zero between launches
+  float* part_o;            // [grid][2][kUnitRows][64] split-piece partial outputs
+  float* part_lse;          // [grid][2][kUnitRows]
   int* status;
   int grid;                 // CTAs of the attention kernel (<= plan.total)
 };
@@ -62,13 +61,14 @@ struct AttnPlan {
 AttnPlan attn_plan(int N, int H, int M);
 
 // Scratch sizes for a given grid.
-inline size_t attn_part_o_floats(int grid) { return (size_t)grid * kUnitRows * kHeadDim; }
-inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * kUnitRows; }
+inline size_t attn_part_o_floats(int grid) { return (size_t)grid * 2 * kUnitRows * kHeadDim; }
+inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kUnitRows; }
 
 cudaError_t attn_setup();                              // kernel attributes (once)
 int attn_ctas_per_sm();                                // resident CTAs per SM
 int attn_smem_bytes();                                 // dynamic shared memory per CTA
-// ev_before / ev_after (may be null) are recorded around the attention kernel.
+// Launches the attention kernel and the merge of split units behind it;
+// ev_before / ev_after (may be null) are recorded around the two.
 cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_before = nullptr,
                              cudaEvent_t ev_after = nullptr);
 

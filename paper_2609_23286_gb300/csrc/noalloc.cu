@@ -27,18 +27,16 @@ namespace {
 constexpr int kMaxCtas = 160;               // split partials for one CTA on each of up to 160 SMs
 constexpr size_t kMaxLse = 262144;          // heads * tokens per frame
 constexpr int kMaxSampled = 8192;           // sampled queries per frame
-constexpr int kMaxUnits = 4096;             // (head, query-tile pair) units
 
 struct NoAllocScratch {
-  float part_o[(size_t)kMaxCtas * kUnitRows * kHeadDim];
-  float part_lse[(size_t)kMaxCtas * kUnitRows];
+  float part_o[(size_t)kMaxCtas * 2 * kUnitRows * kHeadDim];  // first / last piece of each CTA
+  float part_lse[(size_t)kMaxCtas * 2 * kUnitRows];
   float lse[kMaxLse];
   int qidx[kMaxSampled];
-  int counters[kMaxUnits * 2];  // split-piece counters, cleared by every call
   int status;  // device status bits when the caller passes no status word
 };
 
-// 11.8 MB; shared by every call on a device.
+// 22.3 MB; shared by every call on a device.
 static __device__ __align__(256) NoAllocScratch g_scratch;
 
 constexpr int kMaxDevices = 64;
@@ -147,7 +145,6 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
   long long G = (long long)setup.sms * setup.ctas_per_sm;
   if (G > pl.total) G = pl.total;
   if (G > kMaxCtas) return REGMEM_ERR_UNSUPPORTED;  // more CTAs than the partial scratch holds
-  if (pl.units > kMaxUnits) return REGMEM_ERR_UNSUPPORTED;
 
   CUtensorMap tq, tk, tv, tbk, tbv;
   const uint64_t rowb = kHeadDim * 2;
@@ -165,8 +162,6 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
   }
 
   int* st = status ? status : &sc->status;
-  if (cudaMemsetAsync(sc->counters, 0, (size_t)pl.units * 2 * sizeof(int), stream) != cudaSuccess)
-    return REGMEM_ERR_CUDA;
   if (!status && cudaMemsetAsync(&sc->status, 0, sizeof(int), stream) != cudaSuccess)
     return REGMEM_ERR_CUDA;
   sampled_tokens_kernel<<<(nq + 255) / 256, 256, 0, stream>>>(sc->qidx, nq, fd->n_special,
@@ -174,7 +169,7 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
   if (cudaGetLastError() != cudaSuccess) return REGMEM_ERR_CUDA;
 
   const float scale = fd->scale == 0.f ? 1.f / std::sqrt((float)kHeadDim) : fd->scale;
-  AttnArgs a;
+  AttnArgs a = {};
   a.tmQ = &tq;
   a.tmK = &tk;
   a.tmV = &tv;
@@ -188,12 +183,11 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
   a.lse = sc->lse;
   a.part_o = sc->part_o;
   a.part_lse = sc->part_lse;
-  a.counters = sc->counters;
   a.status = st;
   a.grid = (int)G;
   if (launch_attention(a, stream) != cudaSuccess) return REGMEM_ERR_CUDA;
 
-  SalArgs sa;
+  SalArgs sa = {};
   sa.tmK = &tk;
   sa.Q = static_cast<const __nv_bfloat16*>(Q);
   sa.qidx = sc->qidx;

@@ -42,7 +42,6 @@ struct regmem {
   int* qidx = nullptr;        // [nq]
   float* part_o = nullptr;    // split-KV partials
   float* part_lse = nullptr;
-  int* counters = nullptr;    // split-piece counters, [units][2]
   int* head_done = nullptr;   // per-head completion counters of the distributed selection
   uint64_t* adm_lists = nullptr;  // per-(head, key tile) candidate lists, [H][nkt][32]
   int attn_grid = 0;
@@ -177,7 +176,7 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   if (!encode_frame_map(&tq, Q, h->N, h->heads) || !encode_frame_map(&tk, K, h->N, h->heads) ||
       !encode_frame_map(&tv, V, h->N, h->heads))
     return fail(h, REGMEM_ERR_CUDA, "cuTensorMapEncodeTiled failed for the frame tensors");
-  AttnArgs a;
+  AttnArgs a = {};
   a.tmQ = &tq;
   a.tmK = &tk;
   a.tmV = &tv;
@@ -191,7 +190,6 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   a.lse = h->lse;
   a.part_o = h->part_o;
   a.part_lse = h->part_lse;
-  a.counters = h->counters;
   a.status = h->status_dev;
   const AttnPlan pl = attn_plan(h->N, h->heads, M);
   const long long G = pl.total < h->attn_grid ? pl.total : h->attn_grid;
@@ -217,6 +215,7 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   h->prof.attention_ctas_per_sm = h->attn_ctas_per_sm;
   const double L = (double)M + h->N;
   h->prof.launches_attention += 1;
+  h->prof.launches_combine += 1;
   if (timed) {
     h->prof.attention_timed += 1;
     h->prof.attention_flops += 4.0 * h->N * L * kHeadDim * h->heads;
@@ -311,9 +310,6 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
   RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_floats(h->attn_grid) * sizeof(float)));
   RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid) * sizeof(float)));
-  const size_t n_counters = (size_t)attn_plan(N, h->heads, 0).units * 2;
-  RM_CUDA(h, cudaMalloc(&h->counters, n_counters * sizeof(int)));
-  RM_CUDA(h, cudaMemset(h->counters, 0, n_counters * sizeof(int)));
   RM_CUDA(h, cudaMalloc(&h->head_done, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMemset(h->head_done, 0, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMalloc(&h->adm_lists, (size_t)h->heads * ((N + kTile - 1) / kTile) * 32 * sizeof(uint64_t)));
@@ -361,7 +357,7 @@ regmem_status attend_impl(regmem_t* h, int32_t layer, const void* Q, const void*
   CUtensorMap tk;
   if (!encode_frame_map(&tk, K, h->N, h->heads))
     return fail(h, REGMEM_ERR_CUDA, "cuTensorMapEncodeTiled failed for K");
-  SalArgs sa;
+  SalArgs sa = {};
   sa.tmK = &tk;
   sa.Q = static_cast<const __nv_bfloat16*>(Q);
   sa.qidx = h->qidx;
@@ -402,7 +398,7 @@ regmem_status check_admit(regmem_t* h, int32_t layer, int32_t k) {
 
 AdmitArgs admit_args(regmem_t* h, int32_t layer, const void* K, const void* V, float* saliency,
                      int32_t k, int32_t* idx_out) {
-  AdmitArgs a;
+  AdmitArgs a = {};
   a.sal = saliency;
   a.K = static_cast<const __nv_bfloat16*>(K);
   a.V = static_cast<const __nv_bfloat16*>(V);
@@ -695,7 +691,6 @@ void regmem_destroy(regmem_t* h) {
   cudaFree(h->qidx);
   cudaFree(h->part_o);
   cudaFree(h->part_lse);
-  cudaFree(h->counters);
   cudaFree(h->head_done);
   cudaFree(h->adm_lists);
   if (h->status_host) cudaFreeHost(h->status_host);

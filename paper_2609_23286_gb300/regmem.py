@@ -57,7 +57,8 @@ class Profile(ctypes.Structure):
     """regmem_profile."""
     _fields_ = [("launches_attention", ctypes.c_int64),
                 ("launches_saliency", ctypes.c_int64), ("launches_admit", ctypes.c_int64),
-                ("launches_anchor", ctypes.c_int64), ("attention_timed", ctypes.c_int64),
+                ("launches_anchor", ctypes.c_int64), ("launches_combine", ctypes.c_int64),
+                ("attention_timed", ctypes.c_int64),
                 ("attention_ms", ctypes.c_double), ("attention_flops", ctypes.c_double),
                 ("attention_bytes", ctypes.c_double), ("attention_ctas", ctypes.c_int32),
                 ("attention_ctas_per_sm", ctypes.c_int32)]
@@ -67,7 +68,7 @@ class Profile(ctypes.Structure):
 
     def launches(self):
         return (self.launches_attention + self.launches_saliency + self.launches_admit
-                + self.launches_anchor)
+                + self.launches_anchor + self.launches_combine)
 
 
 class RegmemError(RuntimeError):
