@@ -509,7 +509,7 @@ constexpr int CMB_THREADS = 4 * BM;
 constexpr int CMB_MAXP = 4;
 
 __global__ void __launch_bounds__(CMB_THREADS) attn_combine_kernel(const Params p, int G) {
-  __shared__ long long s_slot[64];  // row-0 partial index of each piece, in CTA order
+  __shared__ long long s_slot[kAttnMaxGrid];  // row-0 partial index of each piece, in CTA order
   __shared__ int s_np;
   grid_dep_wait();  // every piece's partial is stored
   grid_dep_launch();
@@ -522,7 +522,7 @@ __global__ void __launch_bounds__(CMB_THREADS) attn_combine_kernel(const Params 
     const int b_lo = cta_of(x0, G, T), b_hi = cta_of(x0 + p.nkv - 1, G, T);
     int np = 0;
     if (b_hi > b_lo) {
-      for (int bb = b_lo; bb <= b_hi && np < 64; ++bb) {
+      for (int bb = b_lo; bb <= b_hi; ++bb) {
         const int which = range_begin(bb, G, T) >= x0 ? 0 : 1;
         s_slot[np++] = ((long long)bb * 2 + which) * UROWS + t * BM;
       }
@@ -641,7 +641,7 @@ int attn_smem_bytes() { return (int)SMEM_BYTES; }
 cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_before,
                              cudaEvent_t ev_after) {
   const Params p = make_params(a);
-  if (a.grid < 1 || (long long)a.grid > p.total) return cudaErrorInvalidValue;
+  if (a.grid < 1 || a.grid > kAttnMaxGrid || (long long)a.grid > p.total) return cudaErrorInvalidValue;
   cudaError_t e;
   if (ev_before && (e = cudaEventRecord(ev_before, s)) != cudaSuccess) return e;
   e = launch_pdl(attn_fwd_kernel, dim3(a.grid), dim3(THREADS), SMEM_BYTES, s, *a.tmQ, *a.tmK, *a.tmV,

@@ -60,6 +60,9 @@ struct AttnPlan {
 };
 AttnPlan attn_plan(int N, int H, int M);
 
+// Largest attention grid: the merge of split units lists at most this many
+// pieces per unit.
+constexpr int kAttnMaxGrid = 256;
 // Scratch sizes for a given grid.
 inline size_t attn_part_o_floats(int grid) { return (size_t)grid * 2 * kUnitRows * kHeadDim; }
 inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kUnitRows; }

@@ -6,6 +6,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -300,7 +301,7 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
 
   const size_t bank_elems = (size_t)h->layers * h->heads * cap * kHeadDim;
   h->attn_ctas_per_sm = attn_ctas_per_sm();
-  h->attn_grid = sms * h->attn_ctas_per_sm;
+  h->attn_grid = std::min(sms * h->attn_ctas_per_sm, kAttnMaxGrid);
   RM_CUDA(h, cudaMalloc(&h->bankK, bank_elems * 2));
   RM_CUDA(h, cudaMalloc(&h->bankV, bank_elems * 2));
   RM_CUDA(h, cudaMemset(h->bankK, 0, bank_elems * 2));

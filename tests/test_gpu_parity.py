@@ -106,6 +106,35 @@ def test_teacher_forced_bank_lengths(M):
         st.close()
 
 
+@pytest.mark.parametrize("H,ns,gh,gw,M", [
+    (1, 1, 8, 8, 20352),   # 160 key tiles on the grid: one or two tiles per CTA
+    (1, 1, 8, 8, 40000),   # one unit split over every CTA of the grid
+    (2, 4, 14, 14, 30000),  # two query tiles per unit, each unit over half the grid
+    (3, 5, 37, 37, 5000),  # eleven query tiles: the last unit of each head has one
+])
+def test_split_units_across_many_ctas(H, ns, gh, gw, M):
+    """Few heads and a long bank: units whose key tiles are spread over many
+    CTAs (more than 64 on a full GB300 grid), merged by the combine kernel."""
+    N = ns + gh * gw
+    st = Stream(1, H, ns, gh, gw, budget=14, max_frames=M // 14 + 2, seed=6)
+    try:
+        g = torch.Generator().manual_seed(M + H)
+        bk = (torch.randn(H, M, 64, generator=g) * 1.3).to(torch.bfloat16)
+        bv = torch.randn(H, M, 64, generator=g).to(torch.bfloat16)
+        st.rm.import_bank(0, bk, bv, M)
+        q, k, v = st.inputs(0, 3)
+        out, sal, lse = st.attend(0, q, k, v)
+        torch.cuda.synchronize()
+        ref = orc.attend_frame(to64(q), to64(k), to64(v), [bk[h].double().numpy() for h in range(H)],
+                               [bv[h].double().numpy() for h in range(H)], 1 / 8,
+                               orc.sampled_query_tokens(ns, gh, gw, 2))
+        check_o(out, ref["O"], f"H={H} N={N} M={M}")
+        check_lse(lse, ref["LSE"], f"H={H} N={N} M={M}")
+        check_saliency(sal, ref["S"], f"H={H} N={N} M={M}")
+    finally:
+        st.close()
+
+
 def test_long_bank_sampled_rows():
     """Config-4 end size: a bank of 29360 rows per head (2000 frames at k = 14).
     O is checked on sampled query rows (the oracle computes rows one by one),
