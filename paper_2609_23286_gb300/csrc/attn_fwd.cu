@@ -25,10 +25,10 @@
 //
 // CTA layout, warp-specialised (12 warps, three warpgroups):
 //   warp 0       TMA producer: both Q tiles of a unit, then K and V tiles
-//                through separate 5-stage rings
-//   warps 1, 2   MMA issuers, one lane each, for query tile 0 and 1 (each
-//                follows only its own warpgroup's hand-offs, so a slower
-//                warpgroup never holds up the other's MMAs); warp 1 owns TMEM
+//                through a 5-stage ring (a stage holds one K and one V tile,
+//                which land on one barrier)
+//   warp 1       Q K^T issuer (one lane) for both query tiles; owns TMEM
+//   warp 2       P V issuer (one lane) for both query tiles
 //   warp 3       idle (completes the control warpgroup, whose register
 //                budget is handed to the softmax warpgroups)
 //   warps 4..7   softmax warpgroup 0 -> query tile 0 of the unit
@@ -41,17 +41,18 @@
 // P V is a TS-MMA (P from TMEM, V MN-major in smem).  Keeping P in TMEM keeps
 // it off shared memory, whose bandwidth the SS-MMA operand reads and the TMA
 // writes already use up.
-// Hand-offs are mbarriers: s_full (MMA -> softmax, S(j) computed), p_ready
-// (softmax -> MMA, P(j) stored and S(j) read), o_done (MMA -> softmax, P V(j)
-// done), K/V full and empty rings and Q full/empty; the empty barriers take
-// one arrival per issuer, and both issuers wait every phase of the full
-// barriers in order.  On GB300 each mbarrier hand-off costs a few hundred
-// cycles of latency (arrive, fence and a fresh wait alike), so a query tile
-// has three per key tile: the softmax waits for S(j), waits for P V(j-1)
-// before overwriting P, and arrives once P(j) is stored.  On that arrival the
-// issuer issues Q K^T(j+1) first (S(j) has been read) and then P V(j); the
-// softmax of the other query tile runs while the tensor core works for this
-// one, so the two warpgroups alternate instead of running in lockstep.
+// Hand-offs are mbarriers, per query tile: s_full (S(j) computed), s_free
+// (S(j) read into registers), p_ready (P(j) stored), o_done (P V(j) done);
+// plus the K/V ring's full/empty barriers (the empty ones take one arrival
+// from each issuer) and Q full/empty.  On GB300 every mbarrier hand-off costs
+// a few hundred cycles of latency, even on a phase that has already
+// completed, so the design keeps them off the critical chain where it can:
+// the softmax releases S as soon as it holds S(j) in registers, and the
+// Q K^T issuer computes S(j+1) while the softmax works on tile j; P is
+// single-buffered, so the softmax waits for P V(j-1) before storing P(j).
+// With separate issuers for Q K^T and P V, a Q K^T is never queued behind
+// the issue of a P V in the same thread (an MMA issue blocks while the
+// tensor core is busy).
 // The softmax uses packed fp32x2 FMA/ADD and three-input max, leaving the
 // exp2 (MUFU) as the dominant instruction stream.
 // The softmax keeps a stale running max and only rescales O when the max
@@ -69,7 +70,7 @@ namespace {
 
 constexpr int BM = kTile, BN = kTile, HD = kHeadDim;
 constexpr int UROWS = kUnitRows;         // query rows per unit (two tiles)
-constexpr int KSTAGES = 5, VSTAGES = 5;
+constexpr int STAGES = 5;  // K/V ring depth (a stage holds one K tile and one V tile)
 constexpr int TILE_BYTES = BM * HD * 2;  // 16 KB bf16 tile
 constexpr int THREADS = 384;
 // Register split: launched at 168 per thread (384 x 168 = 64,512); the
@@ -87,11 +88,11 @@ constexpr uint32_t IDESC_PV = idesc_bf16_f32(128, 64, false, true);
 
 struct Smem {
   uint8_t q[2][TILE_BYTES];
-  uint8_t k[KSTAGES][TILE_BYTES];
-  uint8_t v[VSTAGES][TILE_BYTES];
+  uint8_t k[STAGES][TILE_BYTES];
+  uint8_t v[STAGES][TILE_BYTES];
   uint64_t q_full, q_empty;
-  uint64_t k_full[KSTAGES], k_empty[KSTAGES], v_full[VSTAGES], v_empty[VSTAGES];
-  uint64_t s_full[2], p_ready[2], o_done[2];  // per query tile
+  uint64_t kv_full[STAGES], kv_empty[STAGES];
+  uint64_t s_full[2], s_free[2], p_ready[2], o_done[2];  // per query tile
   uint64_t fin_bar;
   uint32_t tmem_base;
   int abort_flag;
@@ -166,18 +167,15 @@ __global__ void __launch_bounds__(THREADS, 1)
     sm.abort_flag = 0;
     sm.never = 0;
     mbar_init(smem_addr(&sm.q_full), 1);
-    mbar_init(smem_addr(&sm.q_empty), 2);
-    for (int s = 0; s < KSTAGES; ++s) {
-      mbar_init(smem_addr(&sm.k_full[s]), 1);
-      mbar_init(smem_addr(&sm.k_empty[s]), 2);
-    }
-    for (int s = 0; s < VSTAGES; ++s) {
-      mbar_init(smem_addr(&sm.v_full[s]), 1);
-      mbar_init(smem_addr(&sm.v_empty[s]), 2);
+    mbar_init(smem_addr(&sm.q_empty), 1);
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(smem_addr(&sm.kv_full[s]), 1);
+      mbar_init(smem_addr(&sm.kv_empty[s]), 2);
     }
     for (int t = 0; t < 2; ++t) {
       mbar_init(smem_addr(&sm.s_full[t]), 1);
-      mbar_init(smem_addr(&sm.p_ready[t]), BM);  // every softmax thread arrives
+      mbar_init(smem_addr(&sm.s_free[t]), BM);   // every softmax thread arrives
+      mbar_init(smem_addr(&sm.p_ready[t]), BM);
       mbar_init(smem_addr(&sm.o_done[t]), 1);
     }
     mbar_init(smem_addr(&sm.fin_bar), 2);
@@ -203,7 +201,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       prefetch_tmap(&tmV);
       prefetch_tmap(&tmBK);
       prefetch_tmap(&tmBV);
-      int nk = 0, nv = 0, piece = 0;  // K tiles, V tiles, Q pairs issued
+      int nkv = 0, piece = 0;  // K/V tile pairs, Q pairs issued
       bool ok = true;
       for (long long x = x_begin; x < x_end && ok;) {
         const Piece pc = piece_at(p, x, x_end);
@@ -215,45 +213,38 @@ __global__ void __launch_bounds__(THREADS, 1)
         tma_load_3d(smem_addr(sm.q[1]), &tmQ, bq, 0, pc.h, (2 * pc.qp + 1) * BM);
         ++piece;
         for (int j = pc.j0; j < pc.j1 && ok; ++j) {
-          const int ks = nk % KSTAGES;
-          if (nk >= KSTAGES)
-            ok = mbar_wait(smem_addr(&sm.k_empty[ks]), ((nk / KSTAGES) - 1) & 1, abort_flag, WAIT_NS);
+          const int st = nkv % STAGES;
+          if (nkv >= STAGES)
+            ok = mbar_wait(smem_addr(&sm.kv_empty[st]), ((nkv / STAGES) - 1) & 1, abort_flag, WAIT_NS);
           if (!ok) break;
-          const uint32_t bk = smem_addr(&sm.k_full[ks]);
-          mbar_arrive_expect_tx(bk, TILE_BYTES);
-          if (j < p.nb) tma_load_3d(smem_addr(sm.k[ks]), &tmBK, bk, 0, j * BN, pc.h);
-          else tma_load_3d(smem_addr(sm.k[ks]), &tmK, bk, 0, pc.h, (j - p.nb) * BN);
-          ++nk;
-          const int vs = nv % VSTAGES;
-          if (nv >= VSTAGES)
-            ok = mbar_wait(smem_addr(&sm.v_empty[vs]), ((nv / VSTAGES) - 1) & 1, abort_flag, WAIT_NS);
-          if (!ok) break;
-          const uint32_t bv = smem_addr(&sm.v_full[vs]);
-          mbar_arrive_expect_tx(bv, TILE_BYTES);
-          if (j < p.nb) tma_load_3d(smem_addr(sm.v[vs]), &tmBV, bv, 0, j * BN, pc.h);
-          else tma_load_3d(smem_addr(sm.v[vs]), &tmV, bv, 0, pc.h, (j - p.nb) * BN);
-          ++nv;
+          // K and V of the tile land on one barrier: the issuer waits once
+          const uint32_t bkv = smem_addr(&sm.kv_full[st]);
+          mbar_arrive_expect_tx(bkv, 2 * TILE_BYTES);
+          if (j < p.nb) {
+            tma_load_3d(smem_addr(sm.k[st]), &tmBK, bkv, 0, j * BN, pc.h);
+            tma_load_3d(smem_addr(sm.v[st]), &tmBV, bkv, 0, j * BN, pc.h);
+          } else {
+            tma_load_3d(smem_addr(sm.k[st]), &tmK, bkv, 0, pc.h, (j - p.nb) * BN);
+            tma_load_3d(smem_addr(sm.v[st]), &tmV, bkv, 0, pc.h, (j - p.nb) * BN);
+          }
+          ++nkv;
         }
         x += pc.j1 - pc.j0;
       }
       // Every issued copy must land before the CTA exits; the last load into
       // each stage is the only one that can still be in flight.
-      for (int i = nk - KSTAGES > 0 ? nk - KSTAGES : 0; i < nk; ++i)
-        mbar_wait(smem_addr(&sm.k_full[i % KSTAGES]), (i / KSTAGES) & 1, never, DRAIN_NS);
-      for (int i = nv - VSTAGES > 0 ? nv - VSTAGES : 0; i < nv; ++i)
-        mbar_wait(smem_addr(&sm.v_full[i % VSTAGES]), (i / VSTAGES) & 1, never, DRAIN_NS);
+      for (int i = nkv - STAGES > 0 ? nkv - STAGES : 0; i < nkv; ++i)
+        mbar_wait(smem_addr(&sm.kv_full[i % STAGES]), (i / STAGES) & 1, never, DRAIN_NS);
       if (piece > 0) mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, never, DRAIN_NS);
     }
   } else if (warp == 1 || warp == 2) {
     // ================================================================ MMA issuers
+    // Warp 1 issues every Q K^T, warp 2 every P V, each for both query
+    // tiles, so a Q K^T never waits behind the issue of a P V in the same
+    // thread.  Both walk the tiles of the CTA's range in the same order.
     if (lane == 0) {
-      const int t = warp - 1;  // query tile served by this issuer
-      const uint32_t sq = smem_addr(sm.q[t]);
-      const uint32_t d_s = tmem + (t ? TM_S1 : TM_S0), d_p = tmem + (t ? TM_P1 : TM_P0);
-      const uint32_t d_o = tmem + (t ? TM_O1 : TM_O0);
-      const uint32_t b_sfull = smem_addr(&sm.s_full[t]), b_pready = smem_addr(&sm.p_ready[t]);
-      const uint32_t b_odone = smem_addr(&sm.o_done[t]);
-      int npv = 0;  // P V issued for this query tile (= p_ready phases consumed)
+      const bool qk_role = warp == 1;
+      uint32_t ph0 = 0, ph1 = 0;  // s_free (QK) or p_ready (PV) phases consumed, per query tile
       int it = 0, piece = 0;
       bool ok = true;
       for (long long x = x_begin; x < x_end && ok;) {
@@ -261,63 +252,64 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int n = pc.j1 - pc.j0;
         x += n;
         ++piece;
-        // The tile-1 issuer has nothing to compute for a unit without a second
-        // query tile, but it still waits every phase of the shared full
-        // barriers in order (skipping a phase would let a later parity wait
-        // match an older phase) and releases stages by a plain arrival.
-        const bool act = (t == 0) || pc.has1;
-        auto release = [&](uint32_t bar) {
-          if (act) mma_commit(bar);  // arrives once this issuer's MMAs are done
-          else mbar_arrive(bar);
-        };
-        ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, WAIT_NS);
+        const int ntiles = pc.has1 ? 2 : 1;  // query tiles of this unit
         const int t0 = it;  // CTA-local index of the piece's first key tile
         it += n;
-        // Q K^T of key tile jj of the piece into S; its K stage (and, after the
-        // piece's last one, the Q tiles) are released when the MMAs complete.
-        auto issue_qk = [&](int jj) {
-          const int ks = (t0 + jj) % KSTAGES;
-          if (act) {
-            const uint32_t kaddr = smem_addr(sm.k[ks]);
+        if (qk_role) {
+          // Q K^T(j) of query tile t goes out once S(j-1) of that tile has
+          // been read; the Q tiles are released after the piece's last one,
+          // each stage after the Q K^T of both tiles has read its K.
+          ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, WAIT_NS);
+          for (int jj = 0; jj < n && ok; ++jj) {
+            const int tq = t0 + jj, st = tq % STAGES;
+            ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, WAIT_NS);
+            const uint32_t kaddr = smem_addr(sm.k[st]);
+            for (int t = 0; t < ntiles && ok; ++t) {
+              if (jj > 0) {
+                ok = mbar_wait(smem_addr(&sm.s_free[t]), (t ? ph1 : ph0) & 1, abort_flag, WAIT_NS);
+                if (t) ++ph1; else ++ph0;
+                if (!ok) break;
+              }
+              tc_fence_after();
+              const uint32_t sq = smem_addr(sm.q[t]), d_s = tmem + (t ? TM_S1 : TM_S0);
 #pragma unroll
-            for (int kk = 0; kk < HD / 16; ++kk)
-              mma_ss(d_s, sdesc_sw128(sq + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
-            mma_commit(b_sfull);
+              for (int kk = 0; kk < HD / 16; ++kk)
+                mma_ss(d_s, sdesc_sw128(sq + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
+              mma_commit(smem_addr(&sm.s_full[t]));
+            }
+            if (!ok) break;
+            mma_commit(smem_addr(&sm.kv_empty[st]));
           }
-          release(smem_addr(&sm.k_empty[ks]));
-          if (jj + 1 == n) release(smem_addr(&sm.q_empty));
-        };
-        auto wait_k = [&](int jj) {
-          const int tq = t0 + jj;
-          return mbar_wait(smem_addr(&sm.k_full[tq % KSTAGES]), (tq / KSTAGES) & 1, abort_flag, WAIT_NS);
-        };
-        if (ok) ok = wait_k(0);
-        if (ok) {
-          tc_fence_after();
-          issue_qk(0);
-        }
-        // Step jj: once P(jj) is stored (which also means S(jj) has been read),
-        // Q K^T of tile jj+1 goes first, so that the softmax gets its next S
-        // early, then P V of tile jj.
-        for (int jj = 0; jj < n && ok; ++jj) {
-          const int tp = t0 + jj;
-          const int vs = tp % VSTAGES;
-          if (jj + 1 < n) ok = wait_k(jj + 1);
-          if (ok) ok = mbar_wait(smem_addr(&sm.v_full[vs]), (tp / VSTAGES) & 1, abort_flag, WAIT_NS);
-          if (ok && act) ok = mbar_wait(b_pready, npv & 1, abort_flag, WAIT_NS);
-          if (!ok) break;
-          tc_fence_after();
-          if (jj + 1 < n) issue_qk(jj + 1);
-          if (act) {
-            const uint32_t vaddr = smem_addr(sm.v[vs]);
+          mma_commit(smem_addr(&sm.q_empty));
+          // the softmax also arrives on s_free for the piece's last tile; the
+          // next piece's first Q K^T waits for it
+          if (ok) ok = mbar_wait(smem_addr(&sm.s_free[0]), ph0 & 1, abort_flag, WAIT_NS);
+          ++ph0;
+          if (ok && ntiles == 2) {
+            ok = mbar_wait(smem_addr(&sm.s_free[1]), ph1 & 1, abort_flag, WAIT_NS);
+            ++ph1;
+          }
+        } else {
+          // P V(j) of query tile t goes out once P(j) of that tile is stored;
+          // each stage is released after the P V of both tiles has read its V.
+          for (int jj = 0; jj < n && ok; ++jj) {
+            const int st = (t0 + jj) % STAGES;
+            const uint32_t vaddr = smem_addr(sm.v[st]);
+            for (int t = 0; t < ntiles && ok; ++t) {
+              ok = mbar_wait(smem_addr(&sm.p_ready[t]), (t ? ph1 : ph0) & 1, abort_flag, WAIT_NS);
+              if (t) ++ph1; else ++ph0;
+              if (!ok) break;
+              tc_fence_after();
+              const uint32_t d_o = tmem + (t ? TM_O1 : TM_O0), d_p = tmem + (t ? TM_P1 : TM_P0);
 #pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk)  // 16 keys = 8 packed columns of P
-              mma_ts(d_o, d_p + kk * 8, sdesc_sw128(vaddr + kk * 2048), IDESC_PV,
-                     (jj == 0 && kk == 0) ? 0u : 1u);
-            mma_commit(b_odone);
-            ++npv;
+              for (int kk = 0; kk < BN / 16; ++kk)  // 16 keys = 8 packed columns of P
+                mma_ts(d_o, d_p + kk * 8, sdesc_sw128(vaddr + kk * 2048), IDESC_PV,
+                       (jj == 0 && kk == 0) ? 0u : 1u);
+              mma_commit(smem_addr(&sm.o_done[t]));
+            }
+            if (!ok) break;
+            mma_commit(smem_addr(&sm.kv_empty[st]));
           }
-          release(smem_addr(&sm.v_empty[vs]));
         }
       }
       // all issued MMAs finish before TMEM and shared memory are released
@@ -335,7 +327,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t tm_s = tmem + lane_off + (t ? TM_S1 : TM_S0);
     const uint32_t tm_o = tmem + lane_off + (t ? TM_O1 : TM_O0);
     const uint32_t b_sfull = smem_addr(&sm.s_full[t]), b_pready = smem_addr(&sm.p_ready[t]);
-    const uint32_t b_odone = smem_addr(&sm.o_done[t]);
+    const uint32_t b_sfree = smem_addr(&sm.s_free[t]), b_odone = smem_addr(&sm.o_done[t]);
     const uint32_t tm_p = tmem + lane_off + (t ? TM_P1 : TM_P0);
     const float c = p.scale_log2;
     uint32_t s_phase = 0, o_phase = 0;
@@ -347,9 +339,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       tc_fence_after();
       return true;
     };
-    // Per key tile the warpgroup has three hand-offs: it waits for S(j), waits
-    // for P V(j-1) (P is single-buffered), and arrives once P(j) is stored,
-    // which also tells the issuer that S(j) has been read.  Every thread
+    // Per key tile the warpgroup waits for S(j), arrives on s_free once S(j)
+    // is in registers, waits for P V(j-1) (P is single-buffered) before
+    // storing P(j), and arrives on p_ready once P(j) is stored.  Every thread
     // arrives (cheaper than a warp-elected arrival after a warp barrier).
     for (long long x = x_begin; x < x_end && !stop;) {
       const Piece pc = piece_at(p, x, x_end);
@@ -367,6 +359,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         s_phase ^= 1;
         uint32_t sr[128];
         tmem_ld128(tm_s, sr);
+        tc_fence_before();
+        mbar_arrive(b_sfree);  // S may be overwritten by the next Q K^T
         const int valid = tile_valid(p, j);
         if (valid < BN) {
 #pragma unroll
