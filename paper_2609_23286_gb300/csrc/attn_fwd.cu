@@ -28,9 +28,9 @@
 //                through a 5-stage ring (a stage holds one K and one V tile,
 //                which land on one barrier)
 //   warp 1       Q K^T issuer (one lane) for both query tiles; owns TMEM
-//   warp 2       P V issuer (one lane) for both query tiles
-//   warp 3       idle (completes the control warpgroup, whose register
-//                budget is handed to the softmax warpgroups)
+//   warps 2, 3   P V issuers (one lane each) for query tile 0 and 1
+// The control warpgroup (warps 0-3) hands most of its register budget to
+// the softmax warpgroups.
 //   warps 4..7   softmax warpgroup 0 -> query tile 0 of the unit
 //   warps 8..11  softmax warpgroup 1 -> query tile 1 of the unit
 // Each softmax thread owns one query row (its TMEM lane).  Each key tile is
@@ -50,9 +50,10 @@
 // the softmax releases S as soon as it holds S(j) in registers, and the
 // Q K^T issuer computes S(j+1) while the softmax works on tile j; P is
 // single-buffered, so the softmax waits for P V(j-1) before storing P(j).
-// With separate issuers for Q K^T and P V, a Q K^T is never queued behind
-// the issue of a P V in the same thread (an MMA issue blocks while the
-// tensor core is busy).
+// With separate issuers for Q K^T and for each tile's P V, a Q K^T is never
+// queued behind the issue of a P V in the same thread (an MMA issue blocks
+// while the tensor core is busy), and one tile's P V never waits for the
+// other tile's softmax.
 // The softmax uses packed fp32x2 FMA/ADD and three-input max, leaving the
 // exp2 (MUFU) as the dominant instruction stream.
 // The softmax keeps a stale running max and only rescales O when the max
@@ -170,7 +171,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     mbar_init(smem_addr(&sm.q_empty), 1);
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(smem_addr(&sm.kv_full[s]), 1);
-      mbar_init(smem_addr(&sm.kv_empty[s]), 2);
+      mbar_init(smem_addr(&sm.kv_empty[s]), 3);  // one arrival per issuer
     }
     for (int t = 0; t < 2; ++t) {
       mbar_init(smem_addr(&sm.s_full[t]), 1);
@@ -178,7 +179,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       mbar_init(smem_addr(&sm.p_ready[t]), BM);
       mbar_init(smem_addr(&sm.o_done[t]), 1);
     }
-    mbar_init(smem_addr(&sm.fin_bar), 2);
+    mbar_init(smem_addr(&sm.fin_bar), 3);
     fence_barrier_init();
   }
   if (warp == 1) {
@@ -237,13 +238,15 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_wait(smem_addr(&sm.kv_full[i % STAGES]), (i / STAGES) & 1, never, DRAIN_NS);
       if (piece > 0) mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, never, DRAIN_NS);
     }
-  } else if (warp == 1 || warp == 2) {
+  } else {
     // ================================================================ MMA issuers
-    // Warp 1 issues every Q K^T, warp 2 every P V, each for both query
-    // tiles, so a Q K^T never waits behind the issue of a P V in the same
-    // thread.  Both walk the tiles of the CTA's range in the same order.
+    // Warp 1 issues every Q K^T (both query tiles), warp 2 the P V of query
+    // tile 0 and warp 3 that of tile 1, so a Q K^T never waits behind the
+    // issue of a P V in the same thread, and neither P V issuer waits for the
+    // other tile's softmax.  All walk the tiles of the CTA's range in order.
     if (lane == 0) {
       const bool qk_role = warp == 1;
+      const int tpv = warp - 2;  // query tile of a P V issuer
       uint32_t ph0 = 0, ph1 = 0;  // s_free (QK) or p_ready (PV) phases consumed, per query tile
       int it = 0, piece = 0;
       bool ok = true;
@@ -289,26 +292,33 @@ __global__ void __launch_bounds__(THREADS, 1)
             ok = mbar_wait(smem_addr(&sm.s_free[1]), ph1 & 1, abort_flag, WAIT_NS);
             ++ph1;
           }
-        } else {
-          // P V(j) of query tile t goes out once P(j) of that tile is stored;
-          // each stage is released after the P V of both tiles has read its V.
+        } else if (tpv == 0 || pc.has1) {
+          // P V(j) of the query tile goes out once P(j) is stored; the stage
+          // is released when it completes (the last read of its V)
+          const uint32_t b_pready = smem_addr(&sm.p_ready[tpv]), b_odone = smem_addr(&sm.o_done[tpv]);
+          const uint32_t d_o = tmem + (tpv ? TM_O1 : TM_O0), d_p = tmem + (tpv ? TM_P1 : TM_P0);
           for (int jj = 0; jj < n && ok; ++jj) {
             const int st = (t0 + jj) % STAGES;
-            const uint32_t vaddr = smem_addr(sm.v[st]);
-            for (int t = 0; t < ntiles && ok; ++t) {
-              ok = mbar_wait(smem_addr(&sm.p_ready[t]), (t ? ph1 : ph0) & 1, abort_flag, WAIT_NS);
-              if (t) ++ph1; else ++ph0;
-              if (!ok) break;
-              tc_fence_after();
-              const uint32_t d_o = tmem + (t ? TM_O1 : TM_O0), d_p = tmem + (t ? TM_P1 : TM_P0);
-#pragma unroll
-              for (int kk = 0; kk < BN / 16; ++kk)  // 16 keys = 8 packed columns of P
-                mma_ts(d_o, d_p + kk * 8, sdesc_sw128(vaddr + kk * 2048), IDESC_PV,
-                       (jj == 0 && kk == 0) ? 0u : 1u);
-              mma_commit(smem_addr(&sm.o_done[t]));
-            }
+            ok = mbar_wait(b_pready, ph0 & 1, abort_flag, WAIT_NS);
+            ++ph0;
             if (!ok) break;
+            tc_fence_after();
+            const uint32_t vaddr = smem_addr(sm.v[st]);
+#pragma unroll
+            for (int kk = 0; kk < BN / 16; ++kk)  // 16 keys = 8 packed columns of P
+              mma_ts(d_o, d_p + kk * 8, sdesc_sw128(vaddr + kk * 2048), IDESC_PV,
+                     (jj == 0 && kk == 0) ? 0u : 1u);
+            mma_commit(b_odone);
             mma_commit(smem_addr(&sm.kv_empty[st]));
+          }
+        } else {
+          // tile 1 of a unit without one: nothing to compute, but the stage
+          // releases keep their order (an arrival for a stage's next use
+          // only after that use's load has landed)
+          for (int jj = 0; jj < n && ok; ++jj) {
+            const int tq = t0 + jj, st = tq % STAGES;
+            ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, WAIT_NS);
+            if (ok) mbar_arrive(smem_addr(&sm.kv_empty[st]));
           }
         }
       }
