@@ -126,8 +126,21 @@ REGMEM_API regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, co
  *   ERR_CAPACITY if the bank would overflow (nothing is appended).
  * idx_out: optional device int32 [H][k] receiving the admitted token indices
  * (ascending per head); NULL to skip.  On the anchor frame nothing is written.
+ * k equal to the number of candidates admits the whole frame (with
+ * candidates = 1 and budget >= N: the unregulated full-KV stream, every
+ * frame's N rows kept); that case is a plain copy, nothing is ranked.
  * State: the layer must have an attend pending (ERR_STATE). */
 REGMEM_API regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out);
+
+/* Admission without head-specific retention (the ablation of Sec. 4.3,
+ * Table 4, "w/o Head-specific Retention"): instead of each head ranking its
+ * own saliency, one set of k candidate tokens is chosen for all heads, ranked
+ * by the saliency summed over heads (fp32, heads added in ascending order;
+ * the same order as the head mean), ties -> lower token index, and the rows
+ * of those tokens are appended to every head's bank in ascending token order.
+ * idx_out: optional device int32 [k].  Everything else (anchor frame, k
+ * range, capacity, state) as in regmem_admit. */
+REGMEM_API regmem_status regmem_admit_shared(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out);
 
 /* regmem_attend_frame followed by regmem_admit(layer, k, idx_out), in one
  * call: the whole per-frame step of one layer (Eq. 3, the LSE-Saliency of

@@ -19,7 +19,14 @@ What it computes, per frame t, layer l and head h (paper notation):
 * Eq. 6: per head, the k most salient candidate keys are appended to the
   memory; Eq. 4: the first frame's full K/V is the global anchor.
 * Memory growth (Sec. 3.3, Layer-Specific Memory Allocation):
-  ``|M_t| = |M_1| + (t - 1) k``.
+  ``|M_t| = |M_1| + (t - 1) k``, with ``k = floor(gamma N)`` on the layers
+  that admit (Eq. 6) and k = 0 on the anchor-only layers (Eq. 5); Sec. 4.1
+  makes layers 11-17 (1-based) the admitting ones.
+* The selection without head-specific retention (the ablation of Sec. 4.3,
+  Table 4): one set of k tokens for all heads, ranked by the saliency
+  averaged over heads.
+* The unregulated stream (the full-KV memory the paper compares against):
+  every frame's N rows are kept, i.e. k = N over all tokens.
 
 Everything is float64 and unblocked: the score matrix is materialised in full,
 softmax is taken row by row as written, saliency is a plain column sum, and the
@@ -64,6 +71,9 @@ __all__ = [
     "saliency_direct",
     "saliency_lse",
     "topk_admission",
+    "topk_admission_shared",
+    "retention_k",
+    "paper_layer_k",
     "OracleStream",
 ]
 
@@ -139,6 +149,28 @@ def topk_admission(s: np.ndarray, n_special: int, k: int,
     lo = n_special if candidates == "patch" else 0
     order = sorted(range(lo, n), key=lambda j: (-float(s[j]), j))
     return sorted(order[:k])
+
+
+def topk_admission_shared(s: np.ndarray, n_special: int, k: int,
+                          candidates: str = "patch") -> list[int]:
+    """Top-k without head-specific retention (Sec. 4.3, Table 4, first row):
+    the saliency of all heads ``s`` [H, N] is averaged over heads and one set
+    of k tokens is chosen for every head, ordered and tie-broken as in
+    ``topk_admission``."""
+    mean = np.asarray(s, dtype=np.float64).mean(axis=0)
+    return topk_admission(mean, n_special, k, candidates)
+
+
+def retention_k(gamma: float, n_tokens: int) -> int:
+    """k = floor(gamma N), the tokens a frame adds per head (Eq. 6)."""
+    return int(math.floor(gamma * n_tokens))
+
+
+def paper_layer_k(layers: int, k: int) -> list[int]:
+    """Per-layer admission count of the paper's configuration (Sec. 4.1,
+    Eq. 5 / Eq. 6): layers 11-17 (1-based) admit k rows per frame, every other
+    layer keeps only its anchor frame (k = 0)."""
+    return [k if 11 <= layer + 1 <= 17 else 0 for layer in range(layers)]
 
 
 def attend_frame(q, k, v, bank_k, bank_v, scale, qidx):
@@ -233,16 +265,20 @@ class OracleStream:
         return np.array([topk_admission(s[h], self.n_special, kk, self.candidates)
                          for h in range(self.heads)], dtype=np.int64).reshape(self.heads, kk)
 
-    def admit(self, layer: int, kk: int, indices=None) -> np.ndarray:
+    def admit(self, layer: int, kk: int, indices=None, shared: bool = False) -> np.ndarray:
         """Apply Eq. 4 (empty memory: store the whole frame) or Eq. 6 (append
         the top-kk rows per head).  ``indices`` ([H, kk]) teacher-forces the
-        choice.  Returns the appended token indices per head."""
+        choice; ``shared`` takes one head-averaged choice for all heads.
+        Returns the appended token indices per head."""
         k, v, s = self._pending.pop(layer)
         n = k.shape[0]
         if self.memory_len(layer) == 0:
             idx = np.tile(np.arange(n), (self.heads, 1))
         elif indices is not None:
             idx = np.asarray(indices, dtype=np.int64).reshape(self.heads, kk)
+        elif shared:
+            one = topk_admission_shared(s, self.n_special, kk, self.candidates)
+            idx = np.tile(np.asarray(one, dtype=np.int64).reshape(1, kk), (self.heads, 1))
         else:
             idx = np.array([topk_admission(s[h], self.n_special, kk, self.candidates)
                             for h in range(self.heads)],

@@ -9,8 +9,14 @@
 // admit_kernel (any k): one block per head runs the radix selection of
 //   select.cuh over all of the head's candidates.
 //
-// anchor_kernel (Eq. 4): the first frame's K and V rows of every head become
-// the bank's first N rows.
+// admit_shared_kernel (any k): the selection without head-specific
+//   retention (the ablation of Sec. 4.3, Table 4): one index set for all heads,
+//   ranked by the head sum of the saliency (equivalently its head mean).
+//
+// copy_rows_kernel: rows [lo, lo + n) of the frame appended after row M of
+// every head's bank, in token order.  It serves the first frame (Eq. 4: all N
+// rows become the anchor) and an admission of every candidate (k equal to
+// their count, e.g. the unregulated full-KV stream).
 
 #include "kernels.h"
 #include "ptx.cuh"
@@ -65,29 +71,71 @@ __global__ void __launch_bounds__(LT) admit_lists_kernel(AdmitArgs a, int nkt) {
   if (tid == 0) a.done[h] = 0;
 }
 
-__global__ void anchor_kernel(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
-                              __nv_bfloat16* bankV, long long cap, int N, int H) {
+// One block per head: the candidates' head-summed saliency (fp32, heads added
+// in ascending order, so every block forms the same keys) is ranked as in
+// admit_kernel, and the block appends the chosen rows of its own head.
+__global__ void __launch_bounds__(THREADS) admit_shared_kernel(AdmitArgs a) {
+  __shared__ int red[sel::red_words<THREADS>()], ws[WARPS], bc[2];
+  extern __shared__ uint32_t dyn[];  // keys [n], then the admitted positions [k]
+  grid_dep_wait();  // the saliency kernel has finished
+  grid_dep_launch();
+  const int h = blockIdx.x;
+  const int n = a.N - a.cand_lo;
+  uint32_t* keys = dyn;
+  int* ord = reinterpret_cast<int*>(dyn + n);
+  for (int i = threadIdx.x; i < n; i += THREADS) {
+    float sum = 0.f;
+    for (int hh = 0; hh < a.H; ++hh) sum += __ldcg(a.sal + (size_t)hh * a.N + a.cand_lo + i);
+    keys[i] = sel::order_bits(sum);
+  }
+  __syncthreads();
+  sel::select_topk<THREADS>(keys, n, a.k, ord, red, ws, bc);
+  AdmitArgs b = a;
+  b.idx_out = nullptr;  // one index list, written by block 0
+  sel::append_rows<THREADS>(b, h, ord);
+  if (h == 0 && a.idx_out)
+    for (int r = threadIdx.x; r < a.k; r += THREADS) a.idx_out[r] = a.cand_lo + ord[r];
+}
+
+__global__ void copy_rows_kernel(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
+                                 __nv_bfloat16* bankV, long long cap, long long M, int lo, int n,
+                                 int H, int32_t* idx_out, int idx_rows) {
   grid_dep_wait();
   grid_dep_launch();
-  const long long total = (long long)N * H * 8;  // 16-byte chunks per tensor
+  const long long total = (long long)n * H * 8;  // 16-byte chunks per tensor
   for (long long w = blockIdx.x * (long long)blockDim.x + threadIdx.x; w < 2 * total;
        w += (long long)gridDim.x * blockDim.x) {
     const int which = w >= total;
     const long long e = which ? w - total : w;
     const int c = (int)(e & 7);
-    const long long nh = e >> 3;  // n * H + h
-    const int h = (int)(nh % H);
-    const long long n = nh / H;
-    const uint4* src = reinterpret_cast<const uint4*>((which ? V : K) + nh * HD);
-    uint4* dst = reinterpret_cast<uint4*>((which ? bankV : bankK) + ((size_t)h * cap + n) * HD);
+    const long long rh = e >> 3;  // r * H + h
+    const int h = (int)(rh % H);
+    const long long r = rh / H;
+    const uint4* src = reinterpret_cast<const uint4*>((which ? V : K) + ((lo + r) * H + h) * HD);
+    uint4* dst = reinterpret_cast<uint4*>((which ? bankV : bankK) + ((size_t)h * cap + M + r) * HD);
     dst[c] = src[c];
+    if (idx_out && !which && c == 0 && h < idx_rows) idx_out[(size_t)h * n + r] = (int32_t)(lo + r);
   }
+}
+
+// idx_out (optional) receives lo + r for r < n, in `idx_rows` rows of n.
+cudaError_t launch_copy_rows(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
+                             __nv_bfloat16* bankV, long long cap, long long M, int lo, int n, int H,
+                             int32_t* idx_out, int idx_rows, cudaStream_t s) {
+  const long long work = 2LL * n * H * 8;
+  int blocks = (int)((work + 255) / 256);
+  if (blocks > 4096) blocks = 4096;
+  return launch_pdl(copy_rows_kernel, dim3(blocks), dim3(256), 0, s, K, V, bankK, bankV, cap, M, lo, n,
+                    H, idx_out, idx_rows);
 }
 
 }  // namespace
 
 cudaError_t admit_setup() {
-  return cudaFuncSetAttribute(admit_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(admit_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)(2 * kMaxCandidates * sizeof(int)));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(admit_shared_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)(2 * kMaxCandidates * sizeof(int)));
 }
 
@@ -95,6 +143,8 @@ cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s) {
   const int nc = a.N - a.cand_lo;
   if (nc < 1 || nc > kMaxCandidates || a.k < 0 || a.k > nc) return cudaErrorInvalidValue;
   if (a.k == 0) return cudaSuccess;
+  if (a.k == nc)  // every candidate: nothing to rank
+    return launch_copy_rows(a.K, a.V, a.bankK, a.bankV, a.cap, a.M, a.cand_lo, nc, a.H, a.idx_out, a.H, s);
   if (a.k <= sel::kListK && a.lists && a.done) {
     const int nkt = (a.N + LT - 1) / LT;
     return launch_pdl(admit_lists_kernel, dim3(a.H * nkt), dim3(LT), 0, s, a, nkt);
@@ -102,12 +152,18 @@ cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s) {
   return launch_pdl(admit_kernel, dim3(a.H), dim3(THREADS), (size_t)(nc + a.k) * sizeof(int), s, a);
 }
 
+cudaError_t launch_admit_shared(const AdmitArgs& a, cudaStream_t s) {
+  const int nc = a.N - a.cand_lo;
+  if (nc < 1 || nc > kMaxCandidates || a.k < 0 || a.k > nc) return cudaErrorInvalidValue;
+  if (a.k == 0) return cudaSuccess;
+  if (a.k == nc)  // every candidate; one index list
+    return launch_copy_rows(a.K, a.V, a.bankK, a.bankV, a.cap, a.M, a.cand_lo, nc, a.H, a.idx_out, 1, s);
+  return launch_pdl(admit_shared_kernel, dim3(a.H), dim3(THREADS), (size_t)(nc + a.k) * sizeof(int), s, a);
+}
+
 cudaError_t launch_anchor(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
                           __nv_bfloat16* bankV, long long cap, int N, int H, cudaStream_t s) {
-  const long long work = 2LL * N * H * 8;
-  int blocks = (int)((work + 255) / 256);
-  if (blocks > 4096) blocks = 4096;
-  return launch_pdl(anchor_kernel, dim3(blocks), dim3(256), 0, s, K, V, bankK, bankV, cap, N, H);
+  return launch_copy_rows(K, V, bankK, bankV, cap, 0, 0, N, H, nullptr, 0, s);
 }
 
 }  // namespace regmem_dev

@@ -93,7 +93,11 @@ struct AdmitArgs {
   int* done;                // [H]
 };
 cudaError_t admit_setup();
+// Per-head admission (Eq. 6): k rows per head, idx_out [H][k].
 cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s);
+// Admission without head-specific retention: one set of k tokens, ranked by
+// the head sum of the saliency, appended to every head; idx_out [k].
+cudaError_t launch_admit_shared(const AdmitArgs& a, cudaStream_t s);
 // First frame (Eq. 4): bank[h][0:N] = frame rows of head h.
 cudaError_t launch_anchor(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
                           __nv_bfloat16* bankV, long long cap, int N, int H, cudaStream_t s);

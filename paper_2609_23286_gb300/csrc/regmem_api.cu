@@ -564,6 +564,25 @@ regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_o
   return REGMEM_OK;
 }
 
+regmem_status regmem_admit_shared(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out) {
+  regmem_status s = ready(h, layer, true);
+  if (s != REGMEM_OK) return s;
+  if (!h->pending[layer])
+    return fail(h, REGMEM_ERR_STATE, "layer %d has no attend pending", layer);
+  if (idx_out && ((reinterpret_cast<uintptr_t>(idx_out) & 3u) != 0))
+    return fail(h, REGMEM_ERR_ARG, "idx_out must be 4-byte aligned");
+  if (h->len[layer] == 0) return regmem_admit(h, layer, k, nullptr);  // Eq. 4 anchor
+  if ((s = check_admit(h, layer, k)) != REGMEM_OK) return s;
+  if (k > 0) {
+    const AdmitArgs a = admit_args(h, layer, h->pK[layer], h->pV[layer], h->pS[layer], k, idx_out);
+    RM_CUDA(h, launch_admit_shared(a, h->stream));
+    h->prof.launches_admit += 1;
+  }
+  h->len[layer] += k;
+  h->pending[layer] = 0;
+  return REGMEM_OK;
+}
+
 regmem_status regmem_frame_attention(regmem_t* h, const void* Q, const void* K, const void* V,
                                      void* out) {
   regmem_status s = ready(h, 0, false);

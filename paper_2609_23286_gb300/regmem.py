@@ -26,6 +26,7 @@ _SIGNATURES = {
     "regmem_attend_frame": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P]),
     "regmem_attend_frame_host": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P]),
     "regmem_admit": (ctypes.c_int, [_P, _I32, _I32, _P]),
+    "regmem_admit_shared": (ctypes.c_int, [_P, _I32, _I32, _P]),
     "regmem_attend_admit": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, _I32, _P]),
     "regmem_attend_admit_host": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, _I32]),
     "regmem_frame_attention": (ctypes.c_int, [_P, _P, _P, _P, _P]),
@@ -159,6 +160,10 @@ def regmem_admit(h, layer, k, idx_out=None):
     return _check(h, load().regmem_admit(h, layer, k, _ptr(idx_out)))
 
 
+def regmem_admit_shared(h, layer, k, idx_out=None):
+    return _check(h, load().regmem_admit_shared(h, layer, k, _ptr(idx_out)))
+
+
 def regmem_attend_admit(h, layer, Q, K, V, out, saliency, k, idx_out=None):
     return _check(h, load().regmem_attend_admit(h, layer, _ptr(Q), _ptr(K), _ptr(V), _ptr(out),
                                                 _ptr(saliency), k, _ptr(idx_out)))
@@ -264,6 +269,10 @@ class RegMem:
 
     def admit(self, layer, k, idx_out=None):
         return regmem_admit(self.h, layer, k, idx_out)
+
+    def admit_shared(self, layer, k, idx_out=None):
+        """One index set for all heads (no head-specific retention)."""
+        return regmem_admit_shared(self.h, layer, k, idx_out)
 
     def attend_admit(self, layer, Q, K, V, out, saliency, k, idx_out=None):
         return regmem_attend_admit(self.h, layer, Q, K, V, out, saliency, k, idx_out)

@@ -67,12 +67,13 @@ class Stream:
     by the shared seeded generator."""
 
     def __init__(self, layers, heads, n_special, grid_h, grid_w, budget, max_frames, seed,
-                 ds=2, device="cuda"):
+                 ds=2, device="cuda", candidates=0):
         self.L, self.H, self.ns, self.gh, self.gw = layers, heads, n_special, grid_h, grid_w
         self.N = n_special + grid_h * grid_w
         self.budget, self.seed, self.ds, self.device = budget, seed, ds, device
         self.rm = regmem.RegMem(layers, heads, 64, budget)
-        self.rm.set_frame(n_special, grid_h, grid_w, ds=ds, max_frames=max_frames)
+        self.rm.set_frame(n_special, grid_h, grid_w, ds=ds, max_frames=max_frames,
+                          candidates=candidates)
         self.rm.set_stream(torch.cuda.current_stream())
         self.scales = [synth.key_scale(seed, l, self.N, device=device) for l in range(layers)]
 

@@ -1,0 +1,177 @@
+"""Parity of the variants the paper studies around its default configuration,
+through the C ABI against the fp64 oracle:
+
+* selection without head-specific retention (Sec. 4.3, Table 4):
+  regmem_admit_shared;
+* the unregulated full-KV memory the paper compares against (every frame's
+  N rows kept; candidates = all tokens, k = N);
+* the layer-specific allocation of Sec. 4.1 (Eq. 5 layers keep only the
+  anchor, Eq. 6 layers admit k per frame);
+* bank export / import as checkpoint and resume of a stream.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from helpers import Stream, check_indices, check_lse, check_o, check_saliency, to64
+
+pytestmark = pytest.mark.gpu
+
+
+def shared_choice_fp32(sal_gpu: torch.Tensor, n_special: int, k: int) -> list[int]:
+    """The integer decision in the kernel's precision: fp32 head sum of the
+    GPU's own fp32 saliency, heads added in ascending order."""
+    s = sal_gpu.detach().cpu().numpy().astype(np.float32)
+    acc = np.zeros(s.shape[1], dtype=np.float32)
+    for h in range(s.shape[0]):
+        acc = (acc + s[h]).astype(np.float32)
+    return orc.topk_admission(acc.astype(np.float64), n_special, k)
+
+
+@pytest.mark.parametrize("kk", [1, 14, 40])
+def test_shared_admission_matches_oracle(kk):
+    """Head-averaged admission on frame 3 of a VGGT-shaped stream: the chosen
+    set equals the fp32 head-sum ranking of the GPU's saliency, differs from
+    the oracle's fp64 head-mean ranking only inside the tie band, and every
+    head's bank receives the same rows."""
+    H, ns, gh, gw = 16, 5, 37, 37
+    st = Stream(1, H, ns, gh, gw, budget=kk, max_frames=4, seed=31)
+    ref = orc.OracleStream(1, H, 64, ns, gh, gw)
+    try:
+        for t in (1, 2, 3):
+            q, k, v = st.inputs(0, t)
+            out, sal, lse = st.attend(0, q, k, v)
+            idx = torch.full((kk,), -1, dtype=torch.int32, device="cuda")
+            st.rm.admit_shared(0, kk, idx)
+            torch.cuda.synchronize()
+            r = ref.attend(0, to64(q), to64(k), to64(v))
+            check_o(out, r["O"], f"t={t}")
+            check_lse(lse, r["LSE"], f"t={t}")
+            check_saliency(sal, r["S"], f"t={t}")
+            if t == 1:
+                ref.admit(0, kk)
+                continue
+            gi = idx.cpu().numpy().astype(np.int64)
+            assert list(gi) == shared_choice_fp32(sal, ns, kk)
+            want = orc.topk_admission_shared(r["S"], ns, kk)
+            if list(gi) != want:
+                mean = r["S"].mean(axis=0)
+                kth = sorted(mean[want])[0]
+                for j in set(gi) ^ set(want):
+                    assert abs(mean[j] - kth) <= 1e-3 * kth + 1e-7 * len(ref.qidx)
+            ref.admit(0, kk, indices=np.tile(gi, (H, 1)))
+            M = st.N + (t - 2) * kk
+            bk, bv = st.export(0)
+            assert bk.shape[1] == M + kk
+            for h in range(H):
+                assert torch.equal(bk[h, M:], k[gi, h].cpu())
+                assert torch.equal(bv[h, M:], v[gi, h].cpu())
+    finally:
+        st.close()
+
+
+@pytest.mark.parametrize("H,ns,gh,gw,frames", [(2, 5, 8, 8, 6), (16, 5, 37, 37, 3)])
+def test_unregulated_full_kv_stream(H, ns, gh, gw, frames):
+    """The full-KV memory: candidates = all tokens and k = N keep every frame
+    whole (a plain copy, nothing ranked); |M_t| = t N and the banks equal the
+    frames' rows in order; attention over the growing memory matches the
+    oracle frame by frame."""
+    N = ns + gh * gw
+    st = Stream(1, H, ns, gh, gw, budget=N, max_frames=frames, seed=32, candidates=1)
+    ref = orc.OracleStream(1, H, 64, ns, gh, gw, candidates="all")
+    try:
+        for t in range(1, frames + 1):
+            q, k, v = st.inputs(0, t)
+            out, sal, lse, idx = st.attend_admit(0, q, k, v, N)
+            torch.cuda.synchronize()
+            r = ref.attend(0, to64(q), to64(k), to64(v))
+            ref.admit(0, N)
+            check_o(out, r["O"], f"t={t}")
+            check_lse(lse, r["LSE"], f"t={t}")
+            check_saliency(sal, r["S"], f"t={t}")
+            assert st.rm.memory_len(0) == ref.memory_len(0) == t * N
+            if t > 1:
+                assert np.array_equal(idx.cpu().numpy(), np.tile(np.arange(N), (H, 1)))
+        bk, bv = st.export(0)
+        for h in range(H):
+            assert np.array_equal(bk[h].double().numpy(), ref.bank_k[0][h])
+            assert np.array_equal(bv[h].double().numpy(), ref.bank_v[0][h])
+    finally:
+        st.close()
+
+
+def test_paper_layer_split_stream():
+    """Sec. 4.1 / Eq. 5-6 on a 24-layer stream of small frames: layers 11-17
+    admit k per frame, the others keep only the anchor frame; outputs match
+    the oracle and the memory lengths follow |M_t| = N + (t - 1) k_l."""
+    L, H, ns, gh, gw, kk, frames = 24, 2, 5, 8, 8, 3, 4
+    ks = orc.paper_layer_k(L, kk)
+    st = Stream(L, H, ns, gh, gw, budget=kk, max_frames=frames, seed=33)
+    ref = orc.OracleStream(L, H, 64, ns, gh, gw)
+    try:
+        for t in range(1, frames + 1):
+            for layer in range(L):
+                q, k, v = st.inputs(layer, t)
+                out, sal, lse, idx = st.attend_admit(layer, q, k, v, ks[layer])
+                torch.cuda.synchronize()
+                r = ref.attend(layer, to64(q), to64(k), to64(v))
+                if t == 1 or ks[layer] == 0:
+                    ref.admit(layer, ks[layer])
+                else:
+                    gi = idx.cpu().numpy().astype(np.int64)
+                    check_indices(gi, to64(sal), r["S"], ns, ks[layer], len(ref.qidx))
+                    ref.admit(layer, ks[layer], indices=gi)
+                if layer in (0, 10, 16, 17, 23):
+                    check_o(out, r["O"], f"t={t} l={layer}")
+                    check_saliency(sal, r["S"], f"t={t} l={layer}")
+        for layer in range(L):
+            assert st.rm.memory_len(layer) == st.N + (frames - 1) * ks[layer]
+            bk, _ = st.export(layer)
+            for h in range(H):
+                assert np.array_equal(bk[h].double().numpy(), ref.bank_k[layer][h])
+    finally:
+        st.close()
+
+
+def test_checkpoint_resume_is_bit_exact():
+    """Export every layer's bank after frame 3, resume in a fresh handle from
+    the imported banks, and run frames 4-5: outputs, saliency, admitted
+    indices and final banks equal those of the uninterrupted stream bit for
+    bit (the kernels are deterministic)."""
+    L, H, ns, gh, gw, kk = 2, 16, 5, 37, 37, 14
+
+    def run(frames, st, store):
+        for t in frames:
+            for layer in range(L):
+                q, k, v = st.inputs(layer, t)
+                out, sal, lse, idx = st.attend_admit(layer, q, k, v, kk)
+                store[(t, layer)] = (out.cpu(), sal.cpu(), idx.cpu())
+        torch.cuda.synchronize()
+
+    whole, resumed = {}, {}
+    a = Stream(L, H, ns, gh, gw, budget=kk, max_frames=5, seed=34)
+    try:
+        run(range(1, 6), a, whole)
+        final_a = [a.export(layer) for layer in range(L)]
+    finally:
+        a.close()
+    b = Stream(L, H, ns, gh, gw, budget=kk, max_frames=5, seed=34)
+    try:
+        run(range(1, 4), b, resumed)
+        ckpt = [b.export(layer) for layer in range(L)]
+    finally:
+        b.close()
+    c = Stream(L, H, ns, gh, gw, budget=kk, max_frames=5, seed=34)
+    try:
+        for layer, (bk, bv) in enumerate(ckpt):
+            c.rm.import_bank(layer, bk, bv, bk.shape[1])
+        run(range(4, 6), c, resumed)
+        final_c = [c.export(layer) for layer in range(L)]
+    finally:
+        c.close()
+    for key, (o, s, i) in whole.items():
+        o2, s2, i2 = resumed[key]
+        assert torch.equal(o, o2) and torch.equal(s, s2) and torch.equal(i, i2), key
+    for (ka, va), (kc, vc) in zip(final_a, final_c):
+        assert torch.equal(ka, kc) and torch.equal(va, vc)

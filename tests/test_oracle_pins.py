@@ -256,9 +256,68 @@ def check_permutation(mod):
     return np.allclose(o1, o2, atol=1e-13) and np.allclose(l1, l2, atol=1e-13)
 
 
+def check_shared_topk(mod):
+    """Selection without head-specific retention (Sec. 4.3, Table 4): the
+    chosen set equals the rank-based top-k of the plain head average written
+    out in Python (ties included); with one head it is the per-head choice;
+    and on a crafted case where each head prefers a different token, the
+    shared choice is the token both heads rank second."""
+    rng = np.random.default_rng(21)
+    ok = True
+    for trial in range(6):
+        H, N, ns, k = 3, 12, 2, 1 + trial % 4
+        s = np.round(rng.random((H, N)) * 4) / 4  # coarse values: many ties
+        mean = [sum(float(s[h][j]) for h in range(H)) / H for j in range(N)]
+        ok &= mod.topk_admission_shared(s, ns, k) == rank_topk(mean, ns, k)
+        ok &= mod.topk_admission_shared(s[:1], ns, k) == mod.topk_admission(s[0], ns, k)
+    crafted = np.zeros((2, 8))
+    crafted[0, 3], crafted[1, 5] = 10.0, 10.0  # head 0 wants 3, head 1 wants 5
+    crafted[:, 6] = 9.0                        # both rank token 6 second
+    ok &= mod.topk_admission_shared(crafted, 1, 1) == [6]
+    ok &= [mod.topk_admission(crafted[h], 1, 1) for h in range(2)] == [[3], [5]]
+    # a stream with shared admission: every head appends the same tokens
+    H, d, ns_, gh, gw = 2, 4, 1, 3, 3
+    st = mod.OracleStream(1, H, d, ns_, gh, gw)
+    Nn = ns_ + gh * gw
+    for t in range(1, 5):
+        q, kx, v = rand((Nn, H, d), rng), rand((Nn, H, d), rng), rand((Nn, H, d), rng)
+        st.attend(0, q, kx, v)
+        idx = st.admit(0, 2, shared=True)
+        ok &= bool(np.all(idx == idx[0]))
+        ok &= st.memory_len(0) == Nn + (t - 1) * 2
+    return bool(ok)
+
+
+def check_retention(mod):
+    """k = floor(gamma N) (Eq. 6): gamma = 0.01 at N = 1374 keeps 13 tokens,
+    gamma = 0.1 keeps 137; the paper's layer split (Sec. 4.1) makes layers
+    11-17 of 24 (1-based) admit and the other 17 keep only the anchor; and
+    the unregulated memory (every token admitted every frame) holds t N rows
+    after t frames, the frames' rows in order."""
+    ok = mod.retention_k(0.01, 1374) == 13 and mod.retention_k(0.1, 1374) == 137
+    ok &= mod.retention_k(0.001, 1374) == 1 and mod.retention_k(1.0, 69) == 69
+    lk = mod.paper_layer_k(24, 14)
+    ok &= [i + 1 for i, x in enumerate(lk) if x == 14] == list(range(11, 18))
+    ok &= sum(1 for x in lk if x == 0) == 17
+    rng = np.random.default_rng(22)
+    H, d, ns_, gh, gw = 2, 4, 1, 2, 3
+    Nn = ns_ + gh * gw
+    st = mod.OracleStream(1, H, d, ns_, gh, gw, candidates="all")
+    ks = []
+    for t in range(1, 5):
+        q, kx, v = rand((Nn, H, d), rng), rand((Nn, H, d), rng), rand((Nn, H, d), rng)
+        st.attend(0, q, kx, v)
+        st.admit(0, Nn)
+        ks.append(kx)
+        ok &= st.memory_len(0) == t * Nn
+    for h in range(H):
+        ok &= np.array_equal(st.bank_k[0][h], np.concatenate([x[:, h] for x in ks]))
+    return bool(ok)
+
+
 PINS = [check_bruteforce, check_sdpa, check_closed_form, check_uniform, check_mass,
         check_topk, check_sampled_queries, check_stream, check_planted_key,
-        check_permutation]
+        check_permutation, check_shared_topk, check_retention]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -343,7 +402,27 @@ def _sampled_transposed(n_special, grid_h, grid_w, ds, ds_floor=False):
     return orc.sampled_query_tokens(n_special, grid_w, grid_h, ds, ds_floor)
 
 
+def _shared_first_head(s, n_special, k, candidates="patch"):
+    return orc.topk_admission(np.asarray(s)[0], n_special, k, candidates)
+
+
+def _shared_max_over_heads(s, n_special, k, candidates="patch"):
+    return orc.topk_admission(np.asarray(s).max(axis=0), n_special, k, candidates)
+
+
+def _retention_rounds(gamma, n_tokens):
+    return int(round(gamma * n_tokens))
+
+
+def _layer_split_shifted(layers, k):
+    return [k if 10 <= layer + 1 <= 16 else 0 for layer in range(layers)]
+
+
 MUTANTS = {
+    "shared_from_first_head": dict(topk_admission_shared=_shared_first_head),
+    "shared_max_not_mean": dict(topk_admission_shared=_shared_max_over_heads),
+    "retention_rounded": dict(retention_k=_retention_rounds),
+    "layer_split_shifted": dict(paper_layer_k=_layer_split_shifted),
     "wrong_scale": dict(attend_head=_attend_head_wrong_scale),
     "k_v_swapped": dict(attend_head=_attend_head_kv_swapped),
     "lse_missing_max": dict(attend_head=_attend_head_no_max_in_lse),
