@@ -88,10 +88,17 @@ def describe(cfg, name):
     return s
 
 
-def attended_rows(cfg, t):
+def layer_k(cfg, layer):
+    """Rows a frame admits per head in `layer` (Eq. 5 layers: 0)."""
+    ks = cfg.get("k_layers")
+    return ks[layer] if ks else cfg["k"]
+
+
+def attended_rows(cfg, t, layer=None):
     """L = M + N attended by frame t (memory rows before frame t plus N)."""
     N = cfg["ns"] + cfg["gh"] * cfg["gw"]
-    M = 0 if t == 1 else N + (t - 2) * cfg["k"]
+    k = cfg["k"] if layer is None else layer_k(cfg, layer)
+    M = 0 if t == 1 else N + (t - 2) * k
     return M + N
 
 
@@ -293,19 +300,22 @@ def make_pool(cfg, P, seed, device):
 
 def run_frames(rm, cfg, pool, t0, count, out, sal, fa_out=None, two_call=False):
     """Enqueue frames t0 .. t0+count-1 (all layers) through the C ABI: one
-    regmem_attend_admit per layer, or regmem_attend_frame + regmem_admit."""
+    regmem_attend_admit per layer, or regmem_attend_frame + regmem_admit
+    (regmem_admit_shared for the head-averaged selection)."""
     P = len(pool[0])
+    shared = cfg.get("selection") == "head-averaged"
     for t in range(t0, t0 + count):
         for layer in range(cfg["layers"]):
             q, k, v = pool[layer][(t - 1) % P]
+            kk = layer_k(cfg, layer)
             if fa_out is not None:
                 fq, fk, fv = pool[layer][t % P]
                 rm.frame_attention(fq, fk, fv, fa_out)
-            if two_call:
+            if two_call or shared:
                 rm.attend_frame(layer, q, k, v, out, sal)
-                rm.admit(layer, cfg["k"])
+                (rm.admit_shared if shared else rm.admit)(layer, kk)
             else:
-                rm.attend_admit(layer, q, k, v, out, sal, cfg["k"])
+                rm.attend_admit(layer, q, k, v, out, sal, kk)
 
 
 def synthetic_bank(cfg, rows, seed, device):
@@ -349,16 +359,18 @@ def gpu_arm(args, cfg, cfg_name):
     fa_out = torch.empty_like(out) if cfg["fa"] else None
     sal = torch.empty(H, N, dtype=torch.float32, device=dev)
 
-    rm = regmem.RegMem(L, H, 64, cfg["k"])
-    rm.set_frame(cfg["ns"], cfg["gh"], cfg["gw"], ds=2, max_frames=S0 - 1 + max(K, W, 1))
+    budget = max(layer_k(cfg, l) for l in range(L))
+    rm = regmem.RegMem(L, H, 64, budget)
+    rm.set_frame(cfg["ns"], cfg["gh"], cfg["gw"], ds=cfg.get("ds", 2),
+                 max_frames=S0 - 1 + max(K, W, 1), candidates=cfg.get("candidates", 0))
     rm.set_stream(stream)
 
     # Starting later in the stream: each layer's bank holds the rows frame S0
     # would see (synthetic rows), restored again after the warm-up.
     banks = None
     if S0 > 1:
-        M0 = attended_rows(cfg, S0) - N
-        banks = [synthetic_bank(cfg, M0, seed * 7919 + l, dev) for l in range(L)]
+        banks = [synthetic_bank(cfg, attended_rows(cfg, S0, l) - N, seed * 7919 + l, dev)
+                 for l in range(L)]
 
     def restore():
         rm.reset()
@@ -374,7 +386,10 @@ def gpu_arm(args, cfg, cfg_name):
 
     clocks = ClockSampler(local_rank)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    rm.profile_enable(PROFILE_EVERY)
+    # every 8th attention launch; 7th when layers differ (so the sample is not
+    # always the same layers of a 24-layer step)
+    every = PROFILE_EVERY if len({layer_k(cfg, l) for l in range(L)}) == 1 else 7
+    rm.profile_enable(every)
     barrier()
     torch.cuda.synchronize()
     clocks.start()
@@ -388,6 +403,7 @@ def gpu_arm(args, cfg, cfg_name):
     ms_local = ev0.elapsed_time(ev1)
     ms = max_over_ranks(ms_local, dev)
     mem_rows = rm.memory_len(0)
+    mem_rows_layers = [rm.memory_len(l) for l in range(L)]
 
     # e2e: host buffers through the public host-buffer entry point
     e2e = None
@@ -410,7 +426,7 @@ def gpu_arm(args, cfg, cfg_name):
                 if hfa is not None:
                     fq, fk, fv = pool[layer][t % P]
                     rm.frame_attention(fq, fk, fv, fa_out)  # frame-attention layer: device inputs
-                rm.attend_admit_host(layer, q, k, v, hout, hsal, cfg["k"])
+                rm.attend_admit_host(layer, q, k, v, hout, hsal, layer_k(cfg, layer))
         e1.record(stream)
         rm.synchronize()
         barrier()
@@ -438,7 +454,8 @@ def gpu_arm(args, cfg, cfg_name):
         peak_sust, peak_burst, peak_src = 1700.0, 1900.0, "fallback"
     attn_tflops = prof.attention_flops / (prof.attention_ms / 1e3) / 1e12 if prof.attention_ms else 0.0
     attn_ms_mean = prof.attention_ms / max(prof.attention_timed, 1)
-    flops_total = sum(4.0 * N * attended_rows(cfg, t) * 64 * H for t in range(S0, S0 + K)) * L
+    flops_total = sum(4.0 * N * attended_rows(cfg, t, l) * 64 * H
+                      for t in range(S0, S0 + K) for l in range(L))
     if cfg["fa"]:
         flops_total += 4.0 * N * N * 64 * H * L * K
     clk = clocks.summary()
@@ -478,7 +495,7 @@ def gpu_arm(args, cfg, cfg_name):
             "traffic": ATTN_TRAFFIC_BYTES_PER_LAUNCH,
             "traffic_note": ATTN_TRAFFIC_NOTE if ATTN_TRAFFIC_BYTES_PER_LAUNCH else None,
             "launches": prof.attention_timed,
-            "launches_sampled_every": PROFILE_EVERY,
+            "launches_sampled_every": every,
             "launches_total": prof.launches_attention,
             "ctas": prof.attention_ctas,
             "ctas_per_sm": prof.attention_ctas_per_sm,
@@ -492,6 +509,15 @@ def gpu_arm(args, cfg, cfg_name):
         "clocks": clk,
         "e2e": e2e,
     }
+    if cfg.get("variant"):
+        share = line["roofline"]["share_of_step"] or 0.0
+        line["config"]["variant"] = cfg["variant"]
+        line["memory"] = {
+            "bank_rows_per_layer": mem_rows_layers,
+            "bank_bytes": int(sum(mem_rows_layers) * H * 64 * 2 * 2),
+            "bank_rows_law": "N + (t - 1) k_l per layer (t N when every frame is kept)",
+        }
+        line["non_attention_ms_per_layer_frame"] = round((1.0 - share) * ms / K / L, 5)
     if cpu is not None:
         line["cpu_baseline"] = {
             "value": round(cpu["frames_per_s"], 6), "unit": UNIT, "cores": cpu["threads"],
@@ -547,12 +573,54 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--two-call", action="store_true",
                     help="per layer regmem_attend_frame + regmem_admit instead of regmem_attend_admit")
+    ap.add_argument("--frames", type=int, default=0, help="override the config's stream length")
+    # variants the paper studies around its default (each prints the same
+    # JSON line with config.variant and a memory footprint)
+    ap.add_argument("--layer-split", action="store_true",
+                    help="Sec. 4.1: layers 11-17 admit k per frame, the others keep only the anchor")
+    ap.add_argument("--gamma", type=float, default=0.0,
+                    help="retention rate: k = floor(gamma N) on the admitting layers (Eq. 6)")
+    ap.add_argument("--ds", type=int, default=0,
+                    help="query down-sampling window for saliency (default 2, Sec. 3.3)")
+    ap.add_argument("--head-avg", action="store_true",
+                    help="one index set for all heads from the head-averaged saliency (Table 4)")
+    ap.add_argument("--unregulated", action="store_true",
+                    help="full-KV memory: every frame's N rows kept (default 200 frames)")
     args = ap.parse_args(argv)
     if args.warmup < 3 and args.impl == "ours":
         ap.error("--warmup must be >= 3")
     cfg = dict(CONFIGS[args.config])
     if args.layers:
         cfg["layers"] = args.layers
+    if args.frames:
+        cfg["frames"] = args.frames
+    variant = {}
+    N = cfg["ns"] + cfg["gh"] * cfg["gw"]
+    if args.gamma:
+        if not 0.0 < args.gamma <= 1.0:
+            ap.error("--gamma must be in (0, 1]")
+        cfg["k"] = int(math.floor(args.gamma * N))
+        variant["gamma"] = args.gamma
+    if args.unregulated:
+        cfg["k"], cfg["candidates"] = N, 1
+        if not args.frames:
+            cfg["frames"] = 200
+        variant["memory"] = "unregulated full-KV (every frame's N rows kept)"
+    if args.layer_split:
+        cfg["k_layers"] = [cfg["k"] if 11 <= l + 1 <= 17 else 0 for l in range(cfg["layers"])]
+        variant["layer_split"] = "layers 11-17 admit k, the others keep only the anchor (Sec. 4.1)"
+    if args.ds:
+        if args.ds < 1:
+            ap.error("--ds must be >= 1")
+        cfg["ds"] = args.ds
+        variant["ds"] = args.ds
+    if args.head_avg:
+        cfg["selection"] = "head-averaged"
+        variant["selection"] = "head-averaged (one index set for all heads)"
+    if variant:
+        variant["k_per_layer"] = [layer_k(cfg, l) for l in range(cfg["layers"])]
+        cfg["variant"] = variant
+        args.no_cpu_baseline = True  # the oracle baseline models the default stream only
     if args.start_frame < 1:
         ap.error("--start-frame must be >= 1")
     if args.impl == "reference":
