@@ -221,7 +221,7 @@ REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
  * All pointers 16-byte aligned (status 4-byte aligned).
  *
  * Scratch: the kernels' split partials, LSE rows and sampled-query list live
- * in one file-scope device array of 22.3 MB that every GPU which loads this
+ * in one file-scope device array of 11.9 MB that every GPU which loads this
  * library holds until the process exits.  Limits, rejected with
  * REGMEM_ERR_UNSUPPORTED before anything is enqueued: heads * N <= 262144,
  * N <= 65536, sampled queries <= 8192, and the attention grid (one CTA per

@@ -63,6 +63,7 @@
 
 #include "kernels.h"
 #include "ptx.cuh"
+#include "split.cuh"
 
 namespace regmem_dev {
 using namespace ptx;
@@ -110,25 +111,16 @@ struct Params {
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  float* part_o;    // [grid][2][256][64]: partials of each CTA's first / last piece
+  __nv_bfloat16* part_o;  // [grid][2][256][64]: partials of each CTA's first / last piece
   float* part_lse;  // [grid][2][256]
   int* status;
 };
 
-__device__ __forceinline__ long long range_begin(int b, int G, long long T) {
-  return (long long)b * T / G;
-}
+using split::cta_of;
+using split::range_begin;
 
 __device__ __forceinline__ int tile_valid(const Params& p, int j) {
   return j < p.nb ? min(BN, p.M - j * BN) : min(BN, p.N - (j - p.nb) * BN);
-}
-
-// CTA whose range contains global tile x.
-__device__ __forceinline__ int cta_of(long long x, int G, long long T) {
-  long long b = x * G / T;
-  while (b + 1 < G && range_begin((int)b + 1, G, T) <= x) ++b;
-  while (b > 0 && range_begin((int)b, G, T) > x) --b;
-  return (int)b;
 }
 
 // One piece of a CTA's range: unit u, key tiles [j0, j1).
@@ -480,12 +472,20 @@ __global__ void __launch_bounds__(THREADS, 1)
         // attn_combine_kernel merges the unit's pieces
         const int which = (x - n == x_begin) ? 0 : 1;
         const size_t pr = ((size_t)b * 2 + which) * UROWS + t * BM + row;
-        float4* dst = reinterpret_cast<float4*>(p.part_o + pr * HD);
+        // O_p in bf16 (half the bytes the merge reads back), LSE_p in fp32;
+        // the LSE is kept in L2 (evict_last) until the merge reads it
+        const uint64_t pol = l2_policy_evict_last();
+        uint4* dst = reinterpret_cast<uint4*>(p.part_o + pr * HD);
 #pragma unroll
-        for (int c4 = 0; c4 < 16; ++c4)
-          dst[c4] = make_float4(__uint_as_float(orr[c4 * 4 + 0]) * inv_l, __uint_as_float(orr[c4 * 4 + 1]) * inv_l,
-                                __uint_as_float(orr[c4 * 4 + 2]) * inv_l, __uint_as_float(orr[c4 * 4 + 3]) * inv_l);
-        p.part_lse[pr] = lse_val;
+        for (int c8 = 0; c8 < 8; ++c8) {
+          uint4 w;
+          w.x = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 0]) * inv_l, __uint_as_float(orr[c8 * 8 + 1]) * inv_l);
+          w.y = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 2]) * inv_l, __uint_as_float(orr[c8 * 8 + 3]) * inv_l);
+          w.z = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 4]) * inv_l, __uint_as_float(orr[c8 * 8 + 5]) * inv_l);
+          w.w = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 6]) * inv_l, __uint_as_float(orr[c8 * 8 + 7]) * inv_l);
+          dst[c8] = w;
+        }
+        st_global_hint(p.part_lse + pr, lse_val, pol);
       }
     }
   }
@@ -502,97 +502,15 @@ __global__ void __launch_bounds__(THREADS, 1)
   grid_dep_launch();
 }
 
-// Merges the pieces of every split unit: one block per (unit, query tile),
-// four threads per query row (16 of its 64 channels each, so the partial
-// rows are read coalesced), and the loads of up to CMB_MAXP pieces issued
-// together so the merge costs one memory round trip.  Blocks of units
-// finished in one CTA, and second tiles of units that have none, return at
-// once.  Pieces are folded in CTA order, so the result does not depend on
-// which CTA finished first.
+// Merges the pieces of every split unit (split.cuh): block j takes merge
+// job j, tile j & 1 of the unit cut by the boundary between CTAs j / 2 and
+// j / 2 + 1.  2 (G - 1) blocks, two per SM: every block is resident at once.
 constexpr int CMB_THREADS = 4 * BM;
-constexpr int CMB_MAXP = 4;
 
-__global__ void __launch_bounds__(CMB_THREADS) attn_combine_kernel(const Params p, int G) {
-  __shared__ long long s_slot[kAttnMaxGrid];  // row-0 partial index of each piece, in CTA order
-  __shared__ int s_np;
+__global__ void __launch_bounds__(CMB_THREADS, 2) attn_combine_kernel(const SplitLayout lay) {
   grid_dep_wait();  // every piece's partial is stored
   grid_dep_launch();
-  const int u = blockIdx.x >> 1, t = blockIdx.x & 1;
-  const int h = u / p.nqp, qp = u - h * p.nqp;
-  if (t == 1 && 2 * qp + 1 >= p.nqt) return;
-  const long long T = p.total;
-  const long long x0 = (long long)u * p.nkv;
-  if (threadIdx.x == 0) {
-    const int b_lo = cta_of(x0, G, T), b_hi = cta_of(x0 + p.nkv - 1, G, T);
-    int np = 0;
-    if (b_hi > b_lo) {
-      for (int bb = b_lo; bb <= b_hi; ++bb) {
-        const int which = range_begin(bb, G, T) >= x0 ? 0 : 1;
-        s_slot[np++] = ((long long)bb * 2 + which) * UROWS + t * BM;
-      }
-    }
-    s_np = np;
-  }
-  __syncthreads();
-  const int np = s_np;
-  if (np == 0) return;  // finished in one CTA
-  const int row = threadIdx.x >> 2, qtr = threadIdx.x & 3;
-  const int q = (2 * qp + t) * BM + row;
-  float lp[CMB_MAXP];
-  float4 v[CMB_MAXP][4];
-#pragma unroll
-  for (int i = 0; i < CMB_MAXP; ++i) {
-    if (i < np) {
-      const size_t pr = (size_t)s_slot[i] + row;
-      lp[i] = __ldcg(p.part_lse + pr);
-      const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD) + qtr * 4;
-#pragma unroll
-      for (int c = 0; c < 4; ++c) v[i][c] = __ldcg(src + c);
-    }
-  }
-  float m = -INFINITY;
-#pragma unroll
-  for (int i = 0; i < CMB_MAXP; ++i)
-    if (i < np) m = fmaxf(m, lp[i]);
-  for (int i = CMB_MAXP; i < np; ++i) m = fmaxf(m, __ldcg(p.part_lse + (size_t)s_slot[i] + row));
-  float den = 0.f, acc[16];
-#pragma unroll
-  for (int c = 0; c < 16; ++c) acc[c] = 0.f;
-  auto fold = [&](float l, const float4 (&w)[4]) {
-    const float a = ex2((l - m) * 1.4426950408889634f);
-    den += a;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      acc[c * 4 + 0] += w[c].x * a;
-      acc[c * 4 + 1] += w[c].y * a;
-      acc[c * 4 + 2] += w[c].z * a;
-      acc[c * 4 + 3] += w[c].w * a;
-    }
-  };
-#pragma unroll
-  for (int i = 0; i < CMB_MAXP; ++i)
-    if (i < np) fold(lp[i], v[i]);
-  for (int i = CMB_MAXP; i < np; ++i) {  // units cut into more pieces than are prefetched
-    const size_t pr = (size_t)s_slot[i] + row;
-    const float4* src = reinterpret_cast<const float4*>(p.part_o + pr * HD) + qtr * 4;
-    float4 w[4];
-#pragma unroll
-    for (int c = 0; c < 4; ++c) w[c] = __ldcg(src + c);
-    fold(__ldcg(p.part_lse + pr), w);
-  }
-  if (q >= p.N) return;
-  const float inv = 1.f / den;
-  uint4* o = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + h) * HD) + qtr * 2;
-#pragma unroll
-  for (int c8 = 0; c8 < 2; ++c8) {
-    uint4 w4;
-    w4.x = pack_bf16x2(acc[c8 * 8 + 0] * inv, acc[c8 * 8 + 1] * inv);
-    w4.y = pack_bf16x2(acc[c8 * 8 + 2] * inv, acc[c8 * 8 + 3] * inv);
-    w4.z = pack_bf16x2(acc[c8 * 8 + 4] * inv, acc[c8 * 8 + 5] * inv);
-    w4.w = pack_bf16x2(acc[c8 * 8 + 6] * inv, acc[c8 * 8 + 7] * inv);
-    o[c8] = w4;
-  }
-  if (qtr == 0) p.lse[(size_t)h * p.N + q] = m + __logf(den);
+  split::merge_job<CMB_THREADS>(lay, blockIdx.x, threadIdx.x);
 }
 
 Params make_params(const AttnArgs& a) {
@@ -616,6 +534,23 @@ Params make_params(const AttnArgs& a) {
 }
 
 }  // namespace
+
+SplitLayout attn_split_layout(const AttnArgs& a) {
+  const Params p = make_params(a);
+  SplitLayout l;
+  l.total = p.total;
+  l.G = a.grid;
+  l.nkv = p.nkv;
+  l.nqp = p.nqp;
+  l.nqt = p.nqt;
+  l.N = a.N;
+  l.H = a.H;
+  l.part_o = a.part_o;
+  l.part_lse = a.part_lse;
+  l.out = a.out;
+  l.lse = a.lse;
+  return l;
+}
 
 AttnPlan attn_plan(int N, int H, int M) {
   AttnPlan pl;
@@ -651,9 +586,11 @@ cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_b
   e = launch_pdl(attn_fwd_kernel, dim3(a.grid), dim3(THREADS), SMEM_BYTES, s, *a.tmQ, *a.tmK, *a.tmV,
                  *a.tmBK, *a.tmBV, p);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(attn_combine_kernel, dim3((unsigned)(p.total / p.nkv) * 2), dim3(CMB_THREADS), 0, s, p,
-                 a.grid);
-  if (e != cudaSuccess) return e;
+  if (a.grid > 1) {  // with one CTA no unit is split
+    e = launch_pdl(attn_combine_kernel, dim3((unsigned)(2 * (a.grid - 1))), dim3(CMB_THREADS), 0, s,
+                   attn_split_layout(a));
+    if (e != cudaSuccess) return e;
+  }
   if (ev_after && (e = cudaEventRecord(ev_after, s)) != cudaSuccess) return e;
   return cudaSuccess;
 }

@@ -36,6 +36,21 @@ constexpr int kStatusTimeout = 1;    // a bounded wait expired
 constexpr int kStatusSmemAlign = 2;  // dynamic shared memory not 1 KB aligned
 
 // Attention over [bank rows ; frame rows] for every (head, 128-row query tile).
+// The attention's stream-K split, as the merge of split units needs it
+// (split.cuh): CTA b takes tiles [b total / G, (b + 1) total / G) of the
+// (unit, key tile) sequence.
+struct SplitLayout {
+  long long total;        // units * nkv
+  int G;                  // attention CTAs
+  int nkv;                // key tiles per unit
+  int nqp, nqt;           // query-tile pairs (units) per head, query tiles per head
+  int N, H;
+  const __nv_bfloat16* part_o;  // [G][2][kUnitRows][64] piece partials (bf16)
+  const float* part_lse;  // [G][2][kUnitRows]
+  __nv_bfloat16* out;     // [N][H][64]
+  float* lse;             // [H][N]
+};
+
 struct AttnArgs {
   const CUtensorMap* tmQ;   // frame tensors [N][H][64] bf16, box 64x1x128
   const CUtensorMap* tmK;
@@ -46,7 +61,7 @@ struct AttnArgs {
   float scale;
   __nv_bfloat16* out;       // [N][H][64]
   float* lse;               // [H][N]
-  float* part_o;            // [grid][2][kUnitRows][64] split-piece partial outputs
+  __nv_bfloat16* part_o;    // [grid][2][kUnitRows][64] split-piece partial outputs (bf16)
   float* part_lse;          // [grid][2][kUnitRows]
   int* status;
   int grid;                 // CTAs of the attention kernel (<= plan.total)
@@ -64,9 +79,11 @@ AttnPlan attn_plan(int N, int H, int M);
 // pieces per unit.
 constexpr int kAttnMaxGrid = 256;
 // Scratch sizes for a given grid.
-inline size_t attn_part_o_floats(int grid) { return (size_t)grid * 2 * kUnitRows * kHeadDim; }
+inline size_t attn_part_o_elems(int grid) { return (size_t)grid * 2 * kUnitRows * kHeadDim; }
 inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kUnitRows; }
 
+// The split of an attention launch with these arguments.
+SplitLayout attn_split_layout(const AttnArgs& a);
 cudaError_t attn_setup();                              // kernel attributes (once)
 int attn_ctas_per_sm();                                // resident CTAs per SM
 int attn_smem_bytes();                                 // dynamic shared memory per CTA

@@ -41,7 +41,7 @@ struct regmem {
 
   float* lse = nullptr;       // [H][N]
   int* qidx = nullptr;        // [nq]
-  float* part_o = nullptr;    // split-KV partials
+  __nv_bfloat16* part_o = nullptr;  // split-KV partials
   float* part_lse = nullptr;
   int* head_done = nullptr;   // per-head completion counters of the distributed selection
   uint64_t* adm_lists = nullptr;  // per-(head, key tile) candidate lists, [H][nkt][32]
@@ -309,7 +309,7 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   RM_CUDA(h, cudaMalloc(&h->lse, (size_t)h->heads * N * sizeof(float)));
   RM_CUDA(h, cudaMalloc(&h->qidx, q.size() * sizeof(int) + 4));
   RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
-  RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_floats(h->attn_grid) * sizeof(float)));
+  RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_elems(h->attn_grid) * sizeof(__nv_bfloat16)));
   RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid) * sizeof(float)));
   RM_CUDA(h, cudaMalloc(&h->head_done, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMemset(h->head_done, 0, h->heads * sizeof(int)));

@@ -1,0 +1,165 @@
+// The attention's stream-K split and the merge of units cut between CTAs.
+//
+// The (unit, key tile) sequence -- a unit is (head, pair of 128-row query
+// tiles), run over every key tile of [bank ; frame] -- is cut into G
+// contiguous equal ranges, CTA b taking [b T / G, (b + 1) T / G).  A unit cut
+// by a CTA boundary leaves, from each CTA that holds part of it, one
+// normalised partial per query row, (O_p, LSE_p), in the CTA's slot 0 (the
+// unit is the CTA's first piece) or 1 (its last piece), O_p in bf16 and LSE_p
+// in fp32.  The merge of Eq. 3
+// over the pieces is the log-sum-exp combination
+//     LSE = log sum_p exp(LSE_p),   O = sum_p exp(LSE_p - LSE) O_p,
+// folded in CTA order, so the result does not depend on which CTA finished
+// first.  The attention kernel writes the partials; attn_combine_kernel,
+// launched right behind it, merges them.
+
+#pragma once
+
+#include <cuda_bf16.h>
+
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace regmem_dev {
+namespace split {
+
+constexpr int kRows = kTile;            // rows of a query tile
+constexpr int kUnitRowsS = kUnitRows;   // rows of a unit (two tiles)
+constexpr int kMergeThreads = 4;        // threads per row in a merge (16 channels each)
+constexpr int kPrefetch = 2;            // pieces whose loads are issued together
+
+using Layout = SplitLayout;
+
+__host__ __device__ __forceinline__ long long range_begin(int b, int G, long long T) {
+  return (long long)b * T / G;
+}
+
+// CTA whose range contains tile x.
+__device__ __forceinline__ int cta_of(long long x, int G, long long T) {
+  long long b = x * G / T;
+  while (b + 1 < G && range_begin((int)b + 1, G, T) <= x) ++b;
+  while (b > 0 && range_begin((int)b, G, T) > x) --b;
+  return (int)b;
+}
+
+// The CTAs holding a split unit: b_lo .. b_hi, and the slot of b_lo's piece
+// (every later CTA holds the unit as its first piece, slot 0).
+struct Pieces {
+  int b_lo, b_hi, which_lo;
+};
+
+// Row `r` (0..255 within the unit) of piece i (0-based from b_lo) in the
+// partial arrays.
+__device__ __forceinline__ size_t piece_row(const Pieces& pc, int i, int r) {
+  const int bb = pc.b_lo + i;
+  const int which = i == 0 ? pc.which_lo : 0;
+  return ((size_t)bb * 2 + which) * kUnitRowsS + r;
+}
+
+// Merged LSE of row r of a split unit.
+__device__ __forceinline__ float merged_lse(const Layout& s, const Pieces& pc, int r) {
+  const uint64_t pol = ptx::l2_policy_evict_first();
+  const int np = pc.b_hi - pc.b_lo + 1;
+  float m = -INFINITY;
+  for (int i = 0; i < np; ++i) m = fmaxf(m, ptx::ld_global_hint(s.part_lse + piece_row(pc, i, r), pol));
+  float den = 0.f;
+  for (int i = 0; i < np; ++i)
+    den += ptx::ex2((ptx::ld_global_hint(s.part_lse + piece_row(pc, i, r), pol) - m) * 1.4426950408889634f);
+  return m + __logf(den);
+}
+
+// Merges 16 channels (quarter qtr) of row r of tile t of split unit u and
+// writes them to out (bf16); the thread with qtr == 0 also writes the LSE.
+// The bf16 partials add one rounding (relative 2^-9) to the rows of split
+// units before the fp32 fold.
+__device__ __forceinline__ void merge_row(const Layout& s, const Pieces& pc, int u, int t, int r,
+                                          int qtr) {
+  const int h = u / s.nqp, qp = u - h * s.nqp;
+  const int q = (2 * qp + t) * kRows + r;
+  const int ur = t * kRows + r;  // row within the unit
+  const int np = pc.b_hi - pc.b_lo + 1;
+  // the partials were kept in L2 for this read; afterwards they may go
+  const uint64_t pol = ptx::l2_policy_evict_first();
+  float lp[kPrefetch];
+  uint4 v[kPrefetch][2];
+#pragma unroll
+  for (int i = 0; i < kPrefetch; ++i) {
+    if (i < np) {
+      const size_t pr = piece_row(pc, i, ur);
+      lp[i] = ptx::ld_global_hint(s.part_lse + pr, pol);
+      const uint4* src = reinterpret_cast<const uint4*>(s.part_o + pr * kHeadDim) + qtr * 2;
+#pragma unroll
+      for (int c = 0; c < 2; ++c) v[i][c] = __ldcg(src + c);
+    }
+  }
+  float m = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < kPrefetch; ++i)
+    if (i < np) m = fmaxf(m, lp[i]);
+  for (int i = kPrefetch; i < np; ++i) m = fmaxf(m, ptx::ld_global_hint(s.part_lse + piece_row(pc, i, ur), pol));
+  float den = 0.f, acc[16];
+#pragma unroll
+  for (int c = 0; c < 16; ++c) acc[c] = 0.f;
+  auto fold = [&](float l, const uint4 (&w)[2]) {
+    const float a = ptx::ex2((l - m) * 1.4426950408889634f);
+    den += a;
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      const uint32_t ww[4] = {w[c].x, w[c].y, w[c].z, w[c].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        acc[c * 8 + e * 2 + 0] += __uint_as_float(ww[e] << 16) * a;
+        acc[c * 8 + e * 2 + 1] += __uint_as_float(ww[e] & 0xFFFF0000u) * a;
+      }
+    }
+  };
+#pragma unroll
+  for (int i = 0; i < kPrefetch; ++i)
+    if (i < np) fold(lp[i], v[i]);
+  for (int i = kPrefetch; i < np; ++i) {  // units cut into more pieces than are prefetched
+    const size_t pr = piece_row(pc, i, ur);
+    const uint4* src = reinterpret_cast<const uint4*>(s.part_o + pr * kHeadDim) + qtr * 2;
+    uint4 w[2];
+#pragma unroll
+    for (int c = 0; c < 2; ++c) w[c] = __ldcg(src + c);
+    fold(ptx::ld_global_hint(s.part_lse + pr, pol), w);
+  }
+  if (q >= s.N) return;
+  const float inv = 1.f / den;
+  uint4* o = reinterpret_cast<uint4*>(s.out + ((size_t)q * s.H + h) * kHeadDim) + qtr * 2;
+#pragma unroll
+  for (int c8 = 0; c8 < 2; ++c8) {
+    uint4 w4;
+    w4.x = ptx::pack_bf16x2(acc[c8 * 8 + 0] * inv, acc[c8 * 8 + 1] * inv);
+    w4.y = ptx::pack_bf16x2(acc[c8 * 8 + 2] * inv, acc[c8 * 8 + 3] * inv);
+    w4.z = ptx::pack_bf16x2(acc[c8 * 8 + 4] * inv, acc[c8 * 8 + 5] * inv);
+    w4.w = ptx::pack_bf16x2(acc[c8 * 8 + 6] * inv, acc[c8 * 8 + 7] * inv);
+    o[c8] = w4;
+  }
+  if (qtr == 0) s.lse[(size_t)h * s.N + q] = merged_lse(s, pc, ur);
+}
+
+// Merge job j (0 .. 2 (G - 1) - 1): query tile j & 1 of the unit cut by the
+// boundary between CTAs j / 2 and j / 2 + 1, unless that boundary is not
+// strictly inside a unit or an earlier boundary cuts the same unit.  Run by a
+// group of NT threads (thread index tid); every row of the tile is merged.
+template <int NT>
+__device__ __forceinline__ void merge_job(const Layout& s, int j, int tid) {
+  static_assert(NT % kMergeThreads == 0, "whole rows per pass");
+  const int bnd = j / 2 + 1, t = j & 1;
+  const long long xb = range_begin(bnd, s.G, s.total);
+  const int u = (int)(xb / s.nkv);
+  const long long x0 = (long long)u * s.nkv;
+  if (xb == x0 || range_begin(bnd - 1, s.G, s.total) > x0) return;
+  const int qp = u % s.nqp;
+  if (t == 1 && 2 * qp + 1 >= s.nqt) return;
+  Pieces pc;
+  pc.b_lo = bnd - 1;  // the CTA holding the unit's first tile
+  pc.b_hi = cta_of(x0 + s.nkv - 1, s.G, s.total);
+  pc.which_lo = range_begin(pc.b_lo, s.G, s.total) == x0 ? 0 : 1;
+  constexpr int RPP = NT / kMergeThreads;  // rows per pass
+  for (int r = tid / kMergeThreads; r < kRows; r += RPP) merge_row(s, pc, u, t, r, tid % kMergeThreads);
+}
+
+}  // namespace split
+}  // namespace regmem_dev
