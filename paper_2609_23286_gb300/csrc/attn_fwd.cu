@@ -49,7 +49,10 @@
 // completed, so the design keeps them off the critical chain where it can:
 // the softmax releases S as soon as it holds S(j) in registers, and the
 // Q K^T issuer computes S(j+1) while the softmax works on tile j; P is
-// single-buffered, so the softmax waits for P V(j-1) before storing P(j).
+// single-buffered, so the softmax waits for P V(j-1) before storing P(j):
+// the tile's P V issuer, idle until the next p_ready anyway, waits for each
+// P V to complete and publishes the count in a shared word, which the
+// softmax checks with one shared load instead of an mbarrier wait.
 // With separate issuers for Q K^T and for each tile's P V, a Q K^T is never
 // queued behind the issue of a P V in the same thread (an MMA issue blocks
 // while the tensor core is busy), and one tile's P V never waits for the
@@ -85,6 +88,7 @@ constexpr uint32_t TM_S0 = 0, TM_S1 = 128, TM_P0 = 256, TM_P1 = 320, TM_O0 = 384
 constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s: a hung pipeline gives up
 constexpr uint64_t DRAIN_NS = 200000000ull;   // 0.2 s for draining on abort
 constexpr float RESCALE_LOG2 = 8.0f;
+constexpr uint32_t FLAG_ABORT = 0x7fffffffu;  // an issuer gave up
 constexpr uint32_t IDESC_QK = idesc_bf16_f32(128, 128, false, false);
 constexpr uint32_t IDESC_PV = idesc_bf16_f32(128, 64, false, true);
 
@@ -99,6 +103,9 @@ struct Smem {
   uint32_t tmem_base;
   int abort_flag;
   int never;  // always 0: abort word for waits that must not be cut short
+  // P V completions per query tile, published by its P V issuer (the softmax
+  // checks this word instead of the o_done mbarrier)
+  uint32_t flag_o[2];
 };
 // The dynamic shared window is requested 1 KB aligned (128-byte swizzle
 // atoms need it) and checked at run time.
@@ -159,6 +166,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   if (tid == 0) {
     sm.abort_flag = 0;
     sm.never = 0;
+    sm.flag_o[0] = sm.flag_o[1] = 0;
     mbar_init(smem_addr(&sm.q_full), 1);
     mbar_init(smem_addr(&sm.q_empty), 1);
     for (int s = 0; s < STAGES; ++s) {
@@ -288,12 +296,16 @@ __global__ void __launch_bounds__(THREADS, 1)
           // P V(j) of the query tile goes out once P(j) is stored; the stage
           // is released when it completes (the last read of its V)
           const uint32_t b_pready = smem_addr(&sm.p_ready[tpv]), b_odone = smem_addr(&sm.o_done[tpv]);
+          const uint32_t f_pub = smem_addr(&sm.flag_o[tpv]);
           const uint32_t d_o = tmem + (tpv ? TM_O1 : TM_O0), d_p = tmem + (tpv ? TM_P1 : TM_P0);
           for (int jj = 0; jj < n && ok; ++jj) {
             const int st = (t0 + jj) % STAGES;
             ok = mbar_wait(b_pready, ph0 & 1, abort_flag, WAIT_NS);
             ++ph0;
-            if (!ok) break;
+            if (!ok) {
+              st_release_shared(f_pub, FLAG_ABORT);
+              break;
+            }
             tc_fence_after();
             const uint32_t vaddr = smem_addr(sm.v[st]);
 #pragma unroll
@@ -302,6 +314,12 @@ __global__ void __launch_bounds__(THREADS, 1)
                      (jj == 0 && kk == 0) ? 0u : 1u);
             mma_commit(b_odone);
             mma_commit(smem_addr(&sm.kv_empty[st]));
+            // publish P V(jj) once complete (the softmax stores P(jj+1)
+            // after it); nothing else waits on this thread until p_ready
+            const bool done = mbar_wait(b_odone, ph1 & 1, abort_flag, WAIT_NS);
+            ++ph1;
+            ok = done;
+            st_release_shared(f_pub, done ? ph1 : FLAG_ABORT);
           }
         } else {
           // tile 1 of a unit without one: nothing to compute, but the stage
@@ -332,12 +350,31 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t b_sfree = smem_addr(&sm.s_free[t]), b_odone = smem_addr(&sm.o_done[t]);
     const uint32_t tm_p = tmem + lane_off + (t ? TM_P1 : TM_P0);
     const float c = p.scale_log2;
-    uint32_t s_phase = 0, o_phase = 0;
+    const uint32_t f_o = smem_addr(&sm.flag_o[t]);
+    uint32_t s_phase = 0, o_phase = 0;  // s_full parity, P V completions consumed
     bool stop = false;
-    // Waits for a phase; the result is uniform across the warp.
+    // Waits until the issuer has published `target` completions (bounded:
+    // gives up on the abort word or after WAIT_NS).  One shared load per
+    // check; the load is warp-wide, so the result is uniform across the warp.
     auto wait_phase = [&](uint32_t bar, uint32_t parity) -> bool {
       const bool ok = mbar_wait(bar, parity, abort_flag, WAIT_NS);
       if (__any_sync(0xffffffffu, !ok)) return false;
+      tc_fence_after();
+      return true;
+    };
+    auto wait_flag = [&](uint32_t flag, uint32_t target) -> bool {
+      uint32_t v = ld_acquire_shared(flag);
+      if (v < target) {
+        const uint64_t t0 = globaltimer_ns();
+        for (int i = 1; v < target; ++i) {
+          v = ld_acquire_shared(flag);
+          if ((i & 255) == 0 && v < target && (*abort_flag || globaltimer_ns() - t0 > WAIT_NS)) {
+            *abort_flag = 1;
+            return false;
+          }
+        }
+      }
+      if (v == FLAG_ABORT) return false;
       tc_fence_after();
       return true;
     };
@@ -410,11 +447,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         if (jj > 0) {
           // P V(j-1) has read P and added into O
-          if (!wait_phase(b_odone, o_phase)) {
+          if (!wait_flag(f_o, ++o_phase)) {
             stop = true;
             break;
           }
-          o_phase ^= 1;
           if (__any_sync(0xffffffffu, need)) {
             // rare (the max grew by > 2^8): rescale O before P V(j) adds to it
 #pragma unroll 1
@@ -441,11 +477,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       if (stop) break;
       // -------------------------------------------------------------- epilogue
-      if (!wait_phase(b_odone, o_phase)) {  // the last tile's P V
+      if (!wait_flag(f_o, ++o_phase)) {  // the last tile's P V
         stop = true;
         break;
       }
-      o_phase ^= 1;
       uint32_t orr[64];
       tmem_ld64(tm_o, orr);
       tc_fence_before();

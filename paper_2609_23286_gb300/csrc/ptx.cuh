@@ -100,13 +100,14 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 }
 
 
-// Device-scope release increment and acquire load (inter-CTA hand-off).
-__device__ __forceinline__ void red_release_add(int* addr, int v) {
-  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(addr), "r"(v) : "memory");
+// CTA-scope release store / acquire load of a shared-memory word (a hand-off
+// between warps of one CTA that costs one shared-memory access to check).
+__device__ __forceinline__ void st_release_shared(uint32_t addr, uint32_t v) {
+  asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
 }
-__device__ __forceinline__ int ld_acquire(const int* addr) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(addr) : "memory");
+__device__ __forceinline__ uint32_t ld_acquire_shared(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
   return v;
 }
 
