@@ -543,9 +543,10 @@ __global__ void __launch_bounds__(THREADS, 1)
 constexpr int CMB_THREADS = 4 * BM;
 
 __global__ void __launch_bounds__(CMB_THREADS, 2) attn_combine_kernel(const SplitLayout lay) {
+  const split::Job jb = split::prepare_job(lay, blockIdx.x);  // layout only: before the wait
   grid_dep_wait();  // every piece's partial is stored
   grid_dep_launch();
-  split::merge_job<CMB_THREADS>(lay, blockIdx.x, threadIdx.x);
+  split::run_job<CMB_THREADS>(lay, jb, threadIdx.x);
 }
 
 Params make_params(const AttnArgs& a) {

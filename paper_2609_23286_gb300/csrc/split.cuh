@@ -56,18 +56,6 @@ __device__ __forceinline__ size_t piece_row(const Pieces& pc, int i, int r) {
   return ((size_t)bb * 2 + which) * kUnitRowsS + r;
 }
 
-// Merged LSE of row r of a split unit.
-__device__ __forceinline__ float merged_lse(const Layout& s, const Pieces& pc, int r) {
-  const uint64_t pol = ptx::l2_policy_evict_first();
-  const int np = pc.b_hi - pc.b_lo + 1;
-  float m = -INFINITY;
-  for (int i = 0; i < np; ++i) m = fmaxf(m, ptx::ld_global_hint(s.part_lse + piece_row(pc, i, r), pol));
-  float den = 0.f;
-  for (int i = 0; i < np; ++i)
-    den += ptx::ex2((ptx::ld_global_hint(s.part_lse + piece_row(pc, i, r), pol) - m) * 1.4426950408889634f);
-  return m + __logf(den);
-}
-
 // Merges 16 channels (quarter qtr) of row r of tile t of split unit u and
 // writes them to out (bf16); the thread with qtr == 0 also writes the LSE.
 // The bf16 partials add one rounding (relative 2^-9) to the rows of split
@@ -136,29 +124,43 @@ __device__ __forceinline__ void merge_row(const Layout& s, const Pieces& pc, int
     w4.w = ptx::pack_bf16x2(acc[c8 * 8 + 6] * inv, acc[c8 * 8 + 7] * inv);
     o[c8] = w4;
   }
-  if (qtr == 0) s.lse[(size_t)h * s.N + q] = merged_lse(s, pc, ur);
+  if (qtr == 0) s.lse[(size_t)h * s.N + q] = m + __logf(den);
 }
 
 // Merge job j (0 .. 2 (G - 1) - 1): query tile j & 1 of the unit cut by the
 // boundary between CTAs j / 2 and j / 2 + 1, unless that boundary is not
-// strictly inside a unit or an earlier boundary cuts the same unit.  Run by a
-// group of NT threads (thread index tid); every row of the tile is merged.
-template <int NT>
-__device__ __forceinline__ void merge_job(const Layout& s, int j, int tid) {
-  static_assert(NT % kMergeThreads == 0, "whole rows per pass");
-  const int bnd = j / 2 + 1, t = j & 1;
+// strictly inside a unit or an earlier boundary cuts the same unit.
+// prepare_job needs only the layout (it can run before the attention's
+// partials are complete); run_job merges every row of the tile with a group
+// of NT threads (thread index tid).
+struct Job {
+  int u, t;  // u < 0: nothing to merge
+  Pieces pc;
+};
+__device__ __forceinline__ Job prepare_job(const Layout& s, int j) {
+  Job jb;
+  jb.u = -1;
+  const int bnd = j / 2 + 1;
+  jb.t = j & 1;
   const long long xb = range_begin(bnd, s.G, s.total);
   const int u = (int)(xb / s.nkv);
   const long long x0 = (long long)u * s.nkv;
-  if (xb == x0 || range_begin(bnd - 1, s.G, s.total) > x0) return;
+  if (xb == x0 || range_begin(bnd - 1, s.G, s.total) > x0) return jb;
   const int qp = u % s.nqp;
-  if (t == 1 && 2 * qp + 1 >= s.nqt) return;
-  Pieces pc;
-  pc.b_lo = bnd - 1;  // the CTA holding the unit's first tile
-  pc.b_hi = cta_of(x0 + s.nkv - 1, s.G, s.total);
-  pc.which_lo = range_begin(pc.b_lo, s.G, s.total) == x0 ? 0 : 1;
+  if (jb.t == 1 && 2 * qp + 1 >= s.nqt) return jb;
+  jb.u = u;
+  jb.pc.b_lo = bnd - 1;  // the CTA holding the unit's first tile
+  jb.pc.b_hi = cta_of(x0 + s.nkv - 1, s.G, s.total);
+  jb.pc.which_lo = range_begin(jb.pc.b_lo, s.G, s.total) == x0 ? 0 : 1;
+  return jb;
+}
+template <int NT>
+__device__ __forceinline__ void run_job(const Layout& s, const Job& jb, int tid) {
+  static_assert(NT % kMergeThreads == 0, "whole rows per pass");
+  if (jb.u < 0) return;
   constexpr int RPP = NT / kMergeThreads;  // rows per pass
-  for (int r = tid / kMergeThreads; r < kRows; r += RPP) merge_row(s, pc, u, t, r, tid % kMergeThreads);
+  for (int r = tid / kMergeThreads; r < kRows; r += RPP)
+    merge_row(s, jb.pc, jb.u, jb.t, r, tid % kMergeThreads);
 }
 
 }  // namespace split
