@@ -62,12 +62,12 @@ CONFIGS = {
 
 # dram__bytes_read.sum + dram__bytes_write.sum of one attention-kernel launch,
 # from an ncu capture of the launch at the stream's mean attended length
-# (frame 1001 of the 2000-frame stream, L = 16,734: 71.79 MB read + 2.73 MB
+# (frame 1001 of the 2000-frame stream, L = 16,734: 71.75 MB read + 1.95 MB
 # written).  Set back to None whenever the
 # attention kernel changes until it is captured again.
-ATTN_TRAFFIC_BYTES_PER_LAUNCH = None
+ATTN_TRAFFIC_BYTES_PER_LAUNCH = 73.71e6
 ATTN_TRAFFIC_NOTE = ("ncu dram bytes of the frame-1001 launch (mean attended length of the "
-                     "stream); the frame-2000 launch moves 552.5 MB (L2 no longer holds a "
+                     "stream); the frame-2000 launch moves 542.2 MB (L2 no longer holds a "
                      "layer's bank)")
 
 
