@@ -454,6 +454,7 @@ def gpu_arm(args, cfg, cfg_name):
         peak_sust, peak_burst, peak_src = 1700.0, 1900.0, "fallback"
     attn_tflops = prof.attention_flops / (prof.attention_ms / 1e3) / 1e12 if prof.attention_ms else 0.0
     attn_ms_mean = prof.attention_ms / max(prof.attention_timed, 1)
+    merge_ms_mean = prof.merge_ms / max(prof.attention_timed, 1)
     flops_total = sum(4.0 * N * attended_rows(cfg, t, l) * 64 * H
                       for t in range(S0, S0 + K) for l in range(L))
     if cfg["fa"]:
@@ -500,9 +501,11 @@ def gpu_arm(args, cfg, cfg_name):
             "ctas": prof.attention_ctas,
             "ctas_per_sm": prof.attention_ctas_per_sm,
             "mean_launch_ms": round(attn_ms_mean, 5),
+            "merge_mean_ms": round(merge_ms_mean, 5),
             "algorithmic_flops_per_launch": prof.attention_flops / max(prof.attention_timed, 1),
             "algorithmic_bytes_per_launch": prof.attention_bytes / max(prof.attention_timed, 1),
-            "share_of_step": (round(attn_ms_mean * prof.launches_attention / ms_local, 4)
+            # attention kernel plus the merge of split units behind it
+            "share_of_step": (round((attn_ms_mean + merge_ms_mean) * prof.launches_attention / ms_local, 4)
                               if ms_local else None),
         },
         "gpu_launches": launches,

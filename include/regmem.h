@@ -243,8 +243,9 @@ REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_frame_desc* fd
  * Counters cover every kernel this handle launched since the last
  * regmem_profile_enable.  When time_attention is set, CUDA events are
  * recorded on the handle's stream immediately before and after the sampled
- * launches of the attention kernel, and attention_ms is the sum of those
- * event intervals; the other kernels are not bracketed. */
+ * launches of the attention kernel and after the merge of split units that
+ * follows it: attention_ms sums the attention kernel's intervals, merge_ms
+ * the merge's; the other kernels are not bracketed. */
 typedef struct regmem_profile {
   int64_t launches_attention; /* attention kernel (attend and frame attention)  */
   int64_t launches_saliency;  /* LSE-saliency kernel                            */
@@ -252,13 +253,15 @@ typedef struct regmem_profile {
   int64_t launches_anchor;    /* first-frame copy kernel                        */
   int64_t launches_combine;   /* merge of units split between attention CTAs   */
   int64_t attention_timed;    /* attention launches with an event pair          */
-  double attention_ms;        /* summed event time of those launches (attention
-                                 kernel plus the merge of split units)          */
+  double attention_ms;        /* summed event time of those launches (the
+                                 attention kernel alone)                        */
   double attention_flops;     /* algorithmic 4*N*(M+N)*64*H of those launches   */
   double attention_bytes;     /* algorithmic HBM bytes of those launches:
                                  Q, O, K/V of the attended rows, LSE           */
   int32_t attention_ctas;     /* grid of the most recent attention launch      */
   int32_t attention_ctas_per_sm; /* resident attention CTAs per SM (occupancy) */
+  double merge_ms;            /* summed event time of the merges of split units
+                                 behind those launches                          */
 } regmem_profile;
 
 /* Resets the counters; time_attention = n >= 1 also brackets every n-th

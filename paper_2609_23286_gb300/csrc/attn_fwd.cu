@@ -614,7 +614,7 @@ int attn_ctas_per_sm() {
 int attn_smem_bytes() { return (int)SMEM_BYTES; }
 
 cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_before,
-                             cudaEvent_t ev_after) {
+                             cudaEvent_t ev_after, cudaEvent_t ev_merged) {
   const Params p = make_params(a);
   if (a.grid < 1 || a.grid > kAttnMaxGrid || (long long)a.grid > p.total) return cudaErrorInvalidValue;
   cudaError_t e;
@@ -622,12 +622,13 @@ cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_b
   e = launch_pdl(attn_fwd_kernel, dim3(a.grid), dim3(THREADS), SMEM_BYTES, s, *a.tmQ, *a.tmK, *a.tmV,
                  *a.tmBK, *a.tmBV, p);
   if (e != cudaSuccess) return e;
+  if (ev_after && (e = cudaEventRecord(ev_after, s)) != cudaSuccess) return e;
   if (a.grid > 1) {  // with one CTA no unit is split
     e = launch_pdl(attn_combine_kernel, dim3((unsigned)(2 * (a.grid - 1))), dim3(CMB_THREADS), 0, s,
                    attn_split_layout(a));
     if (e != cudaSuccess) return e;
   }
-  if (ev_after && (e = cudaEventRecord(ev_after, s)) != cudaSuccess) return e;
+  if (ev_merged && (e = cudaEventRecord(ev_merged, s)) != cudaSuccess) return e;
   return cudaSuccess;
 }
 

@@ -88,9 +88,10 @@ cudaError_t attn_setup();                              // kernel attributes (onc
 int attn_ctas_per_sm();                                // resident CTAs per SM
 int attn_smem_bytes();                                 // dynamic shared memory per CTA
 // Launches the attention kernel and the merge of split units behind it;
-// ev_before / ev_after (may be null) are recorded around the two.
+// ev_before / ev_after (may be null) are recorded around the attention
+// kernel, ev_merged after the merge.
 cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_before = nullptr,
-                             cudaEvent_t ev_after = nullptr);
+                             cudaEvent_t ev_after = nullptr, cudaEvent_t ev_merged = nullptr);
 
 // Per-head top-k of the candidates' saliency and append to the bank.
 struct AdmitArgs {

@@ -60,7 +60,7 @@ struct regmem {
   regmem_profile prof = {};
   int time_every = 0;          // time every n-th attention launch (0: none)
   long long attn_launch_no = 0;
-  std::vector<cudaEvent_t> ev_ring;  // pairs: [2i] before, [2i+1] after
+  std::vector<cudaEvent_t> ev_ring;  // triples: [3i] before, [3i+1] after the attention, [3i+2] after the merge
   std::vector<int> ev_busy;
   size_t ev_next = 0;
 
@@ -159,14 +159,17 @@ regmem_status ready(regmem_t* h, int layer, bool need_layer) {
 
 constexpr size_t kEventPairs = 256;
 
-// Adds the elapsed time of event pair i to the profile and frees the slot.
+// Adds the elapsed times of event triple i to the profile and frees the slot.
 cudaError_t harvest_pair(regmem_t* h, size_t i) {
-  cudaError_t e = cudaEventSynchronize(h->ev_ring[2 * i + 1]);
+  cudaError_t e = cudaEventSynchronize(h->ev_ring[3 * i + 2]);
   if (e != cudaSuccess) return e;
-  float ms = 0.f;
-  e = cudaEventElapsedTime(&ms, h->ev_ring[2 * i], h->ev_ring[2 * i + 1]);
+  float ms = 0.f, ms2 = 0.f;
+  e = cudaEventElapsedTime(&ms, h->ev_ring[3 * i], h->ev_ring[3 * i + 1]);
+  if (e != cudaSuccess) return e;
+  e = cudaEventElapsedTime(&ms2, h->ev_ring[3 * i + 1], h->ev_ring[3 * i + 2]);
   if (e != cudaSuccess) return e;
   h->prof.attention_ms += ms;
+  h->prof.merge_ms += ms2;
   h->ev_busy[i] = 0;
   return cudaSuccess;
 }
@@ -195,28 +198,29 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   const AttnPlan pl = attn_plan(h->N, h->heads, M);
   const long long G = pl.total < h->attn_grid ? pl.total : h->attn_grid;
   a.grid = (int)G;
-  cudaEvent_t eb = nullptr, ea = nullptr;
+  cudaEvent_t eb = nullptr, ea = nullptr, em = nullptr;
   const bool timed = h->time_every > 0 && h->attn_launch_no % h->time_every == 0;
   ++h->attn_launch_no;
   if (timed) {
     if (h->ev_ring.empty()) {
-      h->ev_ring.resize(2 * kEventPairs);
+      h->ev_ring.resize(3 * kEventPairs);
       h->ev_busy.assign(kEventPairs, 0);
       for (auto& e : h->ev_ring) RM_CUDA(h, cudaEventCreate(&e));
     }
     const size_t i = h->ev_next;
     if (h->ev_busy[i]) RM_CUDA(h, harvest_pair(h, i));
-    eb = h->ev_ring[2 * i];
-    ea = h->ev_ring[2 * i + 1];
+    eb = h->ev_ring[3 * i];
+    ea = h->ev_ring[3 * i + 1];
+    em = h->ev_ring[3 * i + 2];
     h->ev_busy[i] = 1;
     h->ev_next = (i + 1) % kEventPairs;
   }
-  RM_CUDA(h, launch_attention(a, h->stream, eb, ea));
+  RM_CUDA(h, launch_attention(a, h->stream, eb, ea, em));
   h->prof.attention_ctas = a.grid;
   h->prof.attention_ctas_per_sm = h->attn_ctas_per_sm;
   const double L = (double)M + h->N;
   h->prof.launches_attention += 1;
-  h->prof.launches_combine += 1;
+  if (a.grid > 1) h->prof.launches_combine += 1;
   if (timed) {
     h->prof.attention_timed += 1;
     h->prof.attention_flops += 4.0 * h->N * L * kHeadDim * h->heads;
