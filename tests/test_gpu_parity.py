@@ -15,13 +15,13 @@ from paper_2609_23286_gb300 import regmem
 pytestmark = pytest.mark.gpu
 
 
-def run_stream(L, H, ns, gh, gw, k, frames, seed, ds=2, check_every=1, fused=False):
+def run_stream(L, H, ns, gh, gw, k, frames, seed, ds=2, check_every=1, fused=False, candidates=0):
     """Free-running stream on GPU and oracle; the oracle adopts the GPU's
     admitted indices after they pass check_indices, so later frames stay
     comparable.  fused: each step is one regmem_attend_admit call (admission
     inside the saliency kernel) instead of regmem_attend_frame + regmem_admit."""
-    st = Stream(L, H, ns, gh, gw, budget=k, max_frames=frames, seed=seed, ds=ds)
-    ref = orc.OracleStream(L, H, 64, ns, gh, gw, ds=ds)
+    st = Stream(L, H, ns, gh, gw, budget=k, max_frames=frames, seed=seed, ds=ds, candidates=candidates)
+    ref = orc.OracleStream(L, H, 64, ns, gh, gw, ds=ds, candidates="all" if candidates else "patch")
     try:
         for t in range(1, frames + 1):
             for layer in range(L):
@@ -41,7 +41,8 @@ def run_stream(L, H, ns, gh, gw, k, frames, seed, ds=2, check_every=1, fused=Fal
                     ref.admit(layer, k)
                 else:
                     gi = idx.cpu().numpy().astype(np.int64)
-                    check_indices(gi, to64(sal), r["S"], ns, k, len(ref.qidx))
+                    check_indices(gi, to64(sal), r["S"], ns, k, len(ref.qidx),
+                                  "all" if candidates else "patch")
                     ref.admit(layer, k, indices=gi)
                 assert st.rm.memory_len(layer) == ref.memory_len(layer) == st.N + (t - 1) * k
             if t in (1, 2, frames):
@@ -60,6 +61,21 @@ def test_tiny_stream_full_oracle(fused):
     """1 layer, 2 heads, 8x8 patches + 5 specials = 69 tokens, 8 frames, k = 1,
     seed 0: the whole stream against the free-running oracle."""
     run_stream(1, 2, 5, 8, 8, 1, 8, seed=0, fused=fused)
+
+
+@pytest.mark.parametrize("ds", [1, 3, 4])
+def test_query_downsampling_factors(ds):
+    """Sec. 3.3 with other windows (T6's sweep): 13 x 11 patches + 5 specials,
+    4 heads, k = 3, 4 frames; ds = 1 samples every patch query, 3 and 4 keep
+    the partial edge windows of the odd grid."""
+    run_stream(1, 4, 5, 13, 11, 3, 4, seed=12, ds=ds, fused=True)
+
+
+@pytest.mark.parametrize("fused", [False, True])
+def test_all_tokens_as_candidates(fused):
+    """candidates = 1: the special tokens may be admitted too (13 x 11 + 5,
+    4 heads, k = 4, 4 frames)."""
+    run_stream(1, 4, 5, 13, 11, 4, 4, seed=13, fused=fused, candidates=1)
 
 
 def test_vggt_layer_first_frames():
