@@ -158,9 +158,15 @@ REGMEM_API regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const v
                                   const void* V, void* out, float* saliency, int32_t k,
                                   int32_t* idx_out);
 
-/* regmem_attend_admit with HOST buffers (layouts and staging as in
- * regmem_attend_frame_host; no index output).  The device->host copies of
- * out and saliency are complete after regmem_synchronize. */
+/* regmem_attend_admit with HOST buffers (layouts as in
+ * regmem_attend_frame_host; no index output).  Two library-owned staging
+ * sets are used alternately and the copies run on two copy streams of the
+ * handle's own (one each way), ordered against the kernels by events: a
+ * call's host->device copies overlap the previous call's kernels and its
+ * device->host copies the next call's.  Host buffers should be pinned (pageable ones are copied
+ * synchronously by CUDA).  The caller must not modify hostQ/hostK/hostV, nor
+ * read hostOut/hostSaliency, before regmem_synchronize (which waits for both
+ * streams); consecutive calls may reuse the same buffers. */
 REGMEM_API regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* hostQ,
                                        const void* hostK, const void* hostV, void* hostOut,
                                        float* hostSaliency, int32_t k);

@@ -55,6 +55,18 @@ struct regmem {
   __nv_bfloat16* stOut = nullptr;
   float* stSal = nullptr;
   std::vector<__nv_bfloat16*> stK, stV;
+  // regmem_attend_admit_host: two staging sets used alternately, copies in
+  // and out on streams of their own, so one call's copies overlap the
+  // neighbouring calls' kernels
+  struct HostSet {
+    __nv_bfloat16 *q = nullptr, *k = nullptr, *v = nullptr, *out = nullptr;
+    float* sal = nullptr;
+    cudaEvent_t h2d = nullptr, done = nullptr, d2h = nullptr;  // inputs in, kernels done, outputs out
+    bool used = false;
+  } hs[2];
+  unsigned hs_next = 0;
+  cudaStream_t cstream = nullptr;  // host->device copies of the host-buffer path
+  cudaStream_t dstream = nullptr;  // device->host copies
 
   // measurement (regmem_profile_*)
   regmem_profile prof = {};
@@ -523,6 +535,28 @@ regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* h
   return unstage_outputs(h, hostOut, hostSaliency);
 }
 
+namespace {
+
+regmem_status host_set(regmem_t* h, regmem_t::HostSet& hs) {
+  const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
+  const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
+  if (!h->cstream) RM_CUDA(h, cudaStreamCreateWithFlags(&h->cstream, cudaStreamNonBlocking));
+  if (!h->dstream) RM_CUDA(h, cudaStreamCreateWithFlags(&h->dstream, cudaStreamNonBlocking));
+  if (!hs.q) {
+    RM_CUDA(h, cudaMalloc(&hs.q, tbytes));
+    RM_CUDA(h, cudaMalloc(&hs.k, tbytes));
+    RM_CUDA(h, cudaMalloc(&hs.v, tbytes));
+    RM_CUDA(h, cudaMalloc(&hs.out, tbytes));
+    RM_CUDA(h, cudaMalloc(&hs.sal, sbytes));
+    RM_CUDA(h, cudaEventCreateWithFlags(&hs.h2d, cudaEventDisableTiming));
+    RM_CUDA(h, cudaEventCreateWithFlags(&hs.done, cudaEventDisableTiming));
+    RM_CUDA(h, cudaEventCreateWithFlags(&hs.d2h, cudaEventDisableTiming));
+  }
+  return REGMEM_OK;
+}
+
+}  // namespace
+
 regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* hostQ,
                                        const void* hostK, const void* hostV, void* hostOut,
                                        float* hostSaliency, int32_t k) {
@@ -534,11 +568,33 @@ regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* h
     return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
                 layer);
   if (h->len[layer] > 0 && (s = check_admit(h, layer, k)) != REGMEM_OK) return s;
-  if ((s = stage_inputs(h, layer, hostQ, hostK, hostV)) != REGMEM_OK) return s;
-  s = regmem_attend_admit(h, layer, h->stQ, h->stK[layer], h->stV[layer], h->stOut, h->stSal, k,
-                          nullptr);
+  // Staging set b (alternating): its inputs are copied in on the input copy
+  // stream once the kernels of its previous use are done, the kernels run on
+  // the handle's stream once the inputs are in and the previous outputs out,
+  // and the outputs are copied back on the output copy stream.  The two copy
+  // streams are separate so that the next call's inputs need not wait for
+  // this call's outputs: its copies overlap this call's kernels.
+  regmem_t::HostSet& hs = h->hs[h->hs_next & 1];
+  if ((s = host_set(h, hs)) != REGMEM_OK) return s;
+  ++h->hs_next;
+  const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
+  const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
+  if (hs.used) RM_CUDA(h, cudaStreamWaitEvent(h->cstream, hs.done, 0));
+  RM_CUDA(h, cudaMemcpyAsync(hs.q, hostQ, tbytes, cudaMemcpyHostToDevice, h->cstream));
+  RM_CUDA(h, cudaMemcpyAsync(hs.k, hostK, tbytes, cudaMemcpyHostToDevice, h->cstream));
+  RM_CUDA(h, cudaMemcpyAsync(hs.v, hostV, tbytes, cudaMemcpyHostToDevice, h->cstream));
+  RM_CUDA(h, cudaEventRecord(hs.h2d, h->cstream));
+  RM_CUDA(h, cudaStreamWaitEvent(h->stream, hs.h2d, 0));
+  if (hs.used) RM_CUDA(h, cudaStreamWaitEvent(h->stream, hs.d2h, 0));
+  s = regmem_attend_admit(h, layer, hs.q, hs.k, hs.v, hs.out, hs.sal, k, nullptr);
   if (s != REGMEM_OK) return s;
-  return unstage_outputs(h, hostOut, hostSaliency);
+  RM_CUDA(h, cudaEventRecord(hs.done, h->stream));
+  RM_CUDA(h, cudaStreamWaitEvent(h->dstream, hs.done, 0));
+  RM_CUDA(h, cudaMemcpyAsync(hostOut, hs.out, tbytes, cudaMemcpyDeviceToHost, h->dstream));
+  RM_CUDA(h, cudaMemcpyAsync(hostSaliency, hs.sal, sbytes, cudaMemcpyDeviceToHost, h->dstream));
+  RM_CUDA(h, cudaEventRecord(hs.d2h, h->dstream));
+  hs.used = true;
+  return REGMEM_OK;
 }
 
 regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out) {
@@ -671,6 +727,8 @@ regmem_status regmem_synchronize(regmem_t* h) {
     if (cudaSetDevice(h->device) != cudaSuccess)
       return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
     RM_CUDA(h, cudaStreamSynchronize(h->stream));
+    if (h->cstream) RM_CUDA(h, cudaStreamSynchronize(h->cstream));
+    if (h->dstream) RM_CUDA(h, cudaStreamSynchronize(h->dstream));
     RM_CUDA(h, cudaGetLastError());
   }
   return check_device_status(h);
@@ -708,6 +766,8 @@ void regmem_destroy(regmem_t* h) {
   if (h->frame_set) {
     cudaSetDevice(h->device);
     cudaStreamSynchronize(h->stream);
+    if (h->cstream) cudaStreamSynchronize(h->cstream);
+    if (h->dstream) cudaStreamSynchronize(h->dstream);
   }
   cudaFree(h->bankK);
   cudaFree(h->bankV);
@@ -724,6 +784,18 @@ void regmem_destroy(regmem_t* h) {
   for (auto* p : h->stK) cudaFree(p);
   for (auto* p : h->stV) cudaFree(p);
   for (auto e : h->ev_ring) cudaEventDestroy(e);
+  for (auto& hs : h->hs) {
+    cudaFree(hs.q);
+    cudaFree(hs.k);
+    cudaFree(hs.v);
+    cudaFree(hs.out);
+    cudaFree(hs.sal);
+    if (hs.h2d) cudaEventDestroy(hs.h2d);
+    if (hs.done) cudaEventDestroy(hs.done);
+    if (hs.d2h) cudaEventDestroy(hs.d2h);
+  }
+  if (h->cstream) cudaStreamDestroy(h->cstream);
+  if (h->dstream) cudaStreamDestroy(h->dstream);
   delete h;
 }
 
