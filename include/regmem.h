@@ -92,6 +92,30 @@ REGMEM_API regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* 
  * enqueued.  NULL selects the legacy default stream. */
 REGMEM_API regmem_status regmem_set_stream(regmem_t* h, void* stream);
 
+/* on = 1: regmem_attend_admit (and its host-buffer form) runs the saliency
+ * and the admission on a side stream of the handle's own, created at the
+ * lowest stream priority, after the call's attention (an event), so that
+ * they overlap the next layer's attention instead of following it on the
+ * stream.  The attention output `out` is complete in stream order as usual;
+ * `saliency`, `idx_out` and the bank update are complete after
+ * regmem_synchronize, and Q/K/V must stay valid until then.  The next
+ * attend of the same layer is ordered after that layer's side work (the
+ * stream waits on an event; one wait covers all side work so far).  For the
+ * attention's CTAs to go ahead of the side blocks when both wait for SMs,
+ * the stream of regmem_set_stream should have a higher priority than the
+ * lowest.  on = 0 (the default) runs everything on the stream; switching it
+ * off orders the stream after the pending side work.  The two-call path
+ * (regmem_attend_frame + regmem_admit), regmem_export_bank,
+ * regmem_import_bank and regmem_reset order the stream after the pending
+ * side work first.  ERR_ARG unless on is 0 or 1. */
+REGMEM_API regmem_status regmem_set_overlap(regmem_t* h, int32_t on);
+
+/* Orders the stream after all side work enqueued so far (an event wait on
+ * the stream; the host does not block), so that work the caller enqueues
+ * next on the stream sees the saliency, indices and banks of every earlier
+ * call.  Nothing to do without overlap. */
+REGMEM_API regmem_status regmem_join(regmem_t* h);
+
 /* Eq. 3 for one layer and the current frame, fused with LSE-Saliency.
  *   out[n][h][:] = softmax(Q_h K_h^T * scale) V_h over the keys
  *                  [bank rows of (layer, h) ; the frame's N keys]
@@ -159,8 +183,8 @@ REGMEM_API regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const v
                                   int32_t* idx_out);
 
 /* regmem_attend_admit with HOST buffers (layouts as in
- * regmem_attend_frame_host; no index output).  Two library-owned staging
- * sets are used alternately and the copies run on two copy streams of the
+ * regmem_attend_frame_host; no index output).  Three library-owned staging
+ * sets are used in turn and the copies run on two copy streams of the
  * handle's own (one each way), ordered against the kernels by events: a
  * call's host->device copies overlap the previous call's kernels and its
  * device->host copies the next call's.  Host buffers should be pinned (pageable ones are copied
@@ -199,11 +223,14 @@ REGMEM_API regmem_status regmem_import_bank(regmem_t* h, int32_t layer, const vo
                                  const void* hostV, int64_t len);
 
 /* Enqueues a copy of the LSE rows of the most recent attend (any layer):
- * dst is device fp32 [H][N] (natural log). */
+ * dst is device fp32 [H][N] (natural log).  Each layer keeps its own LSE
+ * rows ([layers][H][N] fp32 of scratch), so the side work of one layer can
+ * still read them while the next layer's attention runs. */
 REGMEM_API regmem_status regmem_copy_lse(regmem_t* h, float* dst);
 
-/* Waits for all work enqueued on the handle's stream and reports any device
- * status (REGMEM_ERR_TIMEOUT) or CUDA error. */
+/* Waits for all work enqueued on the handle's stream and on its own side and
+ * copy streams, and reports any device status (REGMEM_ERR_TIMEOUT) or CUDA
+ * error. */
 REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
 
 /* Allocation-free attend step.  The paper has no counterpart: this entry

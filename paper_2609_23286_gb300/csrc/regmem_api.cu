@@ -39,7 +39,8 @@ struct regmem {
   __nv_bfloat16* bankV = nullptr;
   std::vector<CUtensorMap> tmBK, tmBV;
 
-  float* lse = nullptr;       // [H][N]
+  float* lse = nullptr;       // [layers][H][N]: each layer's attention writes its own rows
+  int lse_layer = 0;          // layer of the last attention (regmem_copy_lse)
   int* qidx = nullptr;        // [nq]
   __nv_bfloat16* part_o = nullptr;  // split-KV partials
   float* part_lse = nullptr;
@@ -55,18 +56,32 @@ struct regmem {
   __nv_bfloat16* stOut = nullptr;
   float* stSal = nullptr;
   std::vector<__nv_bfloat16*> stK, stV;
-  // regmem_attend_admit_host: two staging sets used alternately, copies in
+  // regmem_attend_admit_host: three staging sets used in turn, copies in
   // and out on streams of their own, so one call's copies overlap the
-  // neighbouring calls' kernels
+  // neighbouring calls' kernels.  Three, not two: with overlap a set's
+  // inputs are read until the call's side work ends, in the next call's
+  // attention, so the inputs of the call after next go to a third set.
+  static constexpr unsigned kHostSets = 3;
   struct HostSet {
     __nv_bfloat16 *q = nullptr, *k = nullptr, *v = nullptr, *out = nullptr;
     float* sal = nullptr;
     cudaEvent_t h2d = nullptr, done = nullptr, d2h = nullptr;  // inputs in, kernels done, outputs out
     bool used = false;
-  } hs[2];
+  } hs[kHostSets];
   unsigned hs_next = 0;
   cudaStream_t cstream = nullptr;  // host->device copies of the host-buffer path
   cudaStream_t dstream = nullptr;  // device->host copies
+
+  // regmem_set_overlap: the saliency and admission of regmem_attend_admit run
+  // on a side stream of the lowest priority, ordered after the call's
+  // attention (event main_ev); the next attention of a layer whose side work
+  // is still unwaited waits for all side work so far (event side_ev).
+  bool overlap = false;
+  cudaStream_t sstream = nullptr;
+  cudaEvent_t main_ev = nullptr, side_ev = nullptr;
+  long long side_seq = 0;      // side submissions so far (side_ev marks the last)
+  long long covered_seq = 0;   // side submissions the handle's stream has waited for
+  std::vector<long long> side_seq_of;  // per layer: its last side submission
 
   // measurement (regmem_profile_*)
   regmem_profile prof = {};
@@ -186,8 +201,27 @@ cudaError_t harvest_pair(regmem_t* h, size_t i) {
   return cudaSuccess;
 }
 
+float* lse_of(regmem_t* h, int layer) { return h->lse + (size_t)layer * h->heads * h->N; }
+
+// Orders the handle's stream after every side submission so far.
+regmem_status join_side(regmem_t* h) {
+  if (h->side_seq > h->covered_seq) {
+    RM_CUDA(h, cudaStreamWaitEvent(h->stream, h->side_ev, 0));
+    h->covered_seq = h->side_seq;
+  }
+  return REGMEM_OK;
+}
+
 regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K, const void* V,
                             void* out, int M) {
+  // the layer's previous saliency and admission (side stream) read its LSE
+  // rows and append to its bank: they finish before this attention starts.
+  // One wait covers all side work so far, so in a stream of frames only the
+  // first layer of each frame waits.
+  if (h->side_seq_of[layer] > h->covered_seq) {
+    regmem_status s = join_side(h);
+    if (s != REGMEM_OK) return s;
+  }
   CUtensorMap tq, tk, tv;
   if (!encode_frame_map(&tq, Q, h->N, h->heads) || !encode_frame_map(&tk, K, h->N, h->heads) ||
       !encode_frame_map(&tv, V, h->N, h->heads))
@@ -203,7 +237,8 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   a.M = M;
   a.scale = h->scale;
   a.out = static_cast<__nv_bfloat16*>(out);
-  a.lse = h->lse;
+  a.lse = lse_of(h, layer);
+  h->lse_layer = layer;
   a.part_o = h->part_o;
   a.part_lse = h->part_lse;
   a.status = h->status_dev;
@@ -281,6 +316,7 @@ regmem_status regmem_create(regmem_t** out, int32_t layers, int32_t heads, int32
   h->pS.assign(layers, nullptr);
   h->stK.assign(layers, nullptr);
   h->stV.assign(layers, nullptr);
+  h->side_seq_of.assign(layers, 0);
   *out = h;
   return REGMEM_OK;
 }
@@ -322,7 +358,7 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   RM_CUDA(h, cudaMalloc(&h->bankV, bank_elems * 2));
   RM_CUDA(h, cudaMemset(h->bankK, 0, bank_elems * 2));
   RM_CUDA(h, cudaMemset(h->bankV, 0, bank_elems * 2));
-  RM_CUDA(h, cudaMalloc(&h->lse, (size_t)h->heads * N * sizeof(float)));
+  RM_CUDA(h, cudaMalloc(&h->lse, (size_t)h->layers * h->heads * N * sizeof(float)));
   RM_CUDA(h, cudaMalloc(&h->qidx, q.size() * sizeof(int) + 4));
   RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
   RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_elems(h->attn_grid) * sizeof(__nv_bfloat16)));
@@ -356,9 +392,30 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   return REGMEM_OK;
 }
 
+regmem_status regmem_set_overlap(regmem_t* h, int32_t on) {
+  if (!h || (on != 0 && on != 1)) return REGMEM_ERR_ARG;
+  if (!on && h->frame_set && h->side_seq > h->covered_seq) {
+    if (cudaSetDevice(h->device) != cudaSuccess)
+      return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
+    regmem_status s = join_side(h);
+    if (s != REGMEM_OK) return s;
+  }
+  h->overlap = on != 0;
+  return REGMEM_OK;
+}
+
+regmem_status regmem_join(regmem_t* h) {
+  if (!h) return REGMEM_ERR_ARG;
+  if (!h->frame_set || h->side_seq <= h->covered_seq) return REGMEM_OK;
+  if (cudaSetDevice(h->device) != cudaSuccess)
+    return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
+  return join_side(h);
+}
+
 regmem_status regmem_set_stream(regmem_t* h, void* stream) {
   if (!h) return REGMEM_ERR_ARG;
   h->stream = static_cast<cudaStream_t>(stream);
+  h->covered_seq = 0;  // the new stream has waited for no side work yet
   return REGMEM_OK;
 }
 
@@ -367,10 +424,14 @@ namespace {
 // Attention and saliency of one frame on one layer; with `adm` the saliency
 // kernel also runs the admission of adm->k rows per head (fused path).
 regmem_status attend_impl(regmem_t* h, int32_t layer, const void* Q, const void* K, const void* V,
-                          void* out, float* saliency, const AdmitArgs* adm) {
+                          void* out, float* saliency, const AdmitArgs* adm, cudaStream_t sst) {
   const long long M = h->len[layer];
   regmem_status s = run_attention(h, layer, Q, K, V, out, (int)M);
   if (s != REGMEM_OK) return s;
+  if (sst != h->stream) {  // the side work starts once the attention (and its merge) is done
+    RM_CUDA(h, cudaEventRecord(h->main_ev, h->stream));
+    RM_CUDA(h, cudaStreamWaitEvent(sst, h->main_ev, 0));
+  }
   CUtensorMap tk;
   if (!encode_frame_map(&tk, K, h->N, h->heads))
     return fail(h, REGMEM_ERR_CUDA, "cuTensorMapEncodeTiled failed for K");
@@ -379,14 +440,14 @@ regmem_status attend_impl(regmem_t* h, int32_t layer, const void* Q, const void*
   sa.Q = static_cast<const __nv_bfloat16*>(Q);
   sa.qidx = h->qidx;
   sa.nq = h->nq;
-  sa.lse = h->lse;
+  sa.lse = lse_of(h, layer);
   sa.N = h->N;
   sa.H = h->heads;
   sa.scale = h->scale;
   sa.sal = saliency;
   sa.status = h->status_dev;
   sa.adm = adm;
-  RM_CUDA(h, launch_saliency(sa, h->stream));
+  RM_CUDA(h, launch_saliency(sa, sst));
   h->prof.launches_saliency += 1;
   return REGMEM_OK;
 }
@@ -433,6 +494,26 @@ AdmitArgs admit_args(regmem_t* h, int32_t layer, const void* K, const void* V, f
   return a;
 }
 
+// Creates the side stream (lowest priority, so that the attention's CTAs are
+// dispatched ahead of its blocks when both wait for SMs) and its events.
+regmem_status side_stream(regmem_t* h) {
+  if (h->sstream) return REGMEM_OK;
+  int least = 0, greatest = 0;
+  RM_CUDA(h, cudaDeviceGetStreamPriorityRange(&least, &greatest));
+  RM_CUDA(h, cudaStreamCreateWithPriority(&h->sstream, cudaStreamNonBlocking, least));
+  RM_CUDA(h, cudaEventCreateWithFlags(&h->main_ev, cudaEventDisableTiming));
+  RM_CUDA(h, cudaEventCreateWithFlags(&h->side_ev, cudaEventDisableTiming));
+  return REGMEM_OK;
+}
+
+// Marks the end of a layer's side submission on stream sst.
+regmem_status finish_side(regmem_t* h, int layer, cudaStream_t sst) {
+  if (sst == h->stream) return REGMEM_OK;
+  RM_CUDA(h, cudaEventRecord(h->side_ev, sst));
+  h->side_seq_of[layer] = ++h->side_seq;
+  return REGMEM_OK;
+}
+
 }  // namespace
 
 regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, const void* K,
@@ -443,7 +524,10 @@ regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, con
   if (h->pending[layer])
     return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
                 layer);
-  if ((s = attend_impl(h, layer, Q, K, V, out, saliency, nullptr)) != REGMEM_OK) return s;
+  // the two-call path runs on the handle's stream and shares the selection
+  // scratch with side-stream admissions
+  if ((s = join_side(h)) != REGMEM_OK) return s;
+  if ((s = attend_impl(h, layer, Q, K, V, out, saliency, nullptr, h->stream)) != REGMEM_OK) return s;
   h->pending[layer] = 1;
   h->pK[layer] = static_cast<const __nv_bfloat16*>(K);
   h->pV[layer] = static_cast<const __nv_bfloat16*>(V);
@@ -462,28 +546,34 @@ regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, con
                 layer);
   if (idx_out && ((reinterpret_cast<uintptr_t>(idx_out) & 3u) != 0))
     return fail(h, REGMEM_ERR_ARG, "idx_out must be 4-byte aligned");
+  cudaStream_t sst = h->stream;  // stream of the saliency and admission
+  if (h->overlap) {
+    if ((s = side_stream(h)) != REGMEM_OK) return s;
+    sst = h->sstream;
+  }
   if (h->len[layer] == 0) {  // Eq. 4: the first frame is kept whole
-    if ((s = attend_impl(h, layer, Q, K, V, out, saliency, nullptr)) != REGMEM_OK) return s;
+    if ((s = attend_impl(h, layer, Q, K, V, out, saliency, nullptr, sst)) != REGMEM_OK) return s;
     auto* bk = h->bankK + (size_t)layer * h->heads * h->cap * kHeadDim;
     auto* bv = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
     RM_CUDA(h, launch_anchor(static_cast<const __nv_bfloat16*>(K), static_cast<const __nv_bfloat16*>(V),
-                             bk, bv, h->cap, h->N, h->heads, h->stream));
+                             bk, bv, h->cap, h->N, h->heads, sst));
     h->prof.launches_anchor += 1;
     h->len[layer] = h->N;
-    return REGMEM_OK;
+    return finish_side(h, layer, sst);
   }
   if ((s = check_admit(h, layer, k)) != REGMEM_OK) return s;
   const AdmitArgs a = admit_args(h, layer, K, V, saliency, k, idx_out);
   // k <= 32: the admission runs inside the saliency kernel; larger k takes
   // the separate single-block selection
   const bool fused = k > 0 && k <= kFusedMaxK;
-  if ((s = attend_impl(h, layer, Q, K, V, out, saliency, fused ? &a : nullptr)) != REGMEM_OK) return s;
+  if ((s = attend_impl(h, layer, Q, K, V, out, saliency, fused ? &a : nullptr, sst)) != REGMEM_OK)
+    return s;
   if (k > 0 && !fused) {
-    RM_CUDA(h, launch_admit(a, h->stream));
+    RM_CUDA(h, launch_admit(a, sst));
     h->prof.launches_admit += 1;
   }
   h->len[layer] += k;
-  return REGMEM_OK;
+  return finish_side(h, layer, sst);
 }
 
 namespace {
@@ -568,27 +658,34 @@ regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* h
     return fail(h, REGMEM_ERR_STATE, "layer %d already has an attend pending; call regmem_admit",
                 layer);
   if (h->len[layer] > 0 && (s = check_admit(h, layer, k)) != REGMEM_OK) return s;
-  // Staging set b (alternating): its inputs are copied in on the input copy
+  // Staging set b (in turn): its inputs are copied in on the input copy
   // stream once the kernels of its previous use are done, the kernels run on
   // the handle's stream once the inputs are in and the previous outputs out,
   // and the outputs are copied back on the output copy stream.  The two copy
   // streams are separate so that the next call's inputs need not wait for
   // this call's outputs: its copies overlap this call's kernels.
-  regmem_t::HostSet& hs = h->hs[h->hs_next & 1];
+  regmem_t::HostSet& hs = h->hs[h->hs_next % regmem_t::kHostSets];
   if ((s = host_set(h, hs)) != REGMEM_OK) return s;
   ++h->hs_next;
   const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
   const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
-  if (hs.used) RM_CUDA(h, cudaStreamWaitEvent(h->cstream, hs.done, 0));
+  // The input copy stream also waits for the set's previous output copies,
+  // so that the handle's stream needs one event wait per call (each wait
+  // between two kernels costs the launch overlap of the second).
+  if (hs.used) {
+    RM_CUDA(h, cudaStreamWaitEvent(h->cstream, hs.done, 0));
+    RM_CUDA(h, cudaStreamWaitEvent(h->cstream, hs.d2h, 0));
+  }
   RM_CUDA(h, cudaMemcpyAsync(hs.q, hostQ, tbytes, cudaMemcpyHostToDevice, h->cstream));
   RM_CUDA(h, cudaMemcpyAsync(hs.k, hostK, tbytes, cudaMemcpyHostToDevice, h->cstream));
   RM_CUDA(h, cudaMemcpyAsync(hs.v, hostV, tbytes, cudaMemcpyHostToDevice, h->cstream));
   RM_CUDA(h, cudaEventRecord(hs.h2d, h->cstream));
   RM_CUDA(h, cudaStreamWaitEvent(h->stream, hs.h2d, 0));
-  if (hs.used) RM_CUDA(h, cudaStreamWaitEvent(h->stream, hs.d2h, 0));
   s = regmem_attend_admit(h, layer, hs.q, hs.k, hs.v, hs.out, hs.sal, k, nullptr);
   if (s != REGMEM_OK) return s;
-  RM_CUDA(h, cudaEventRecord(hs.done, h->stream));
+  // with overlap the call ends on the side stream (its saliency and
+  // admission follow the attention there)
+  RM_CUDA(h, cudaEventRecord(hs.done, h->overlap ? h->sstream : h->stream));
   RM_CUDA(h, cudaStreamWaitEvent(h->dstream, hs.done, 0));
   RM_CUDA(h, cudaMemcpyAsync(hostOut, hs.out, tbytes, cudaMemcpyDeviceToHost, h->dstream));
   RM_CUDA(h, cudaMemcpyAsync(hostSaliency, hs.sal, sbytes, cudaMemcpyDeviceToHost, h->dstream));
@@ -655,6 +752,12 @@ regmem_status regmem_frame_attention(regmem_t* h, const void* Q, const void* K, 
 
 regmem_status regmem_reset(regmem_t* h) {
   if (!h) return REGMEM_ERR_ARG;
+  if (h->frame_set && h->side_seq > h->covered_seq) {  // the new stream's writes follow the old side work
+    if (cudaSetDevice(h->device) != cudaSuccess)
+      return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
+    regmem_status s = join_side(h);
+    if (s != REGMEM_OK) return s;
+  }
   for (int l = 0; l < h->layers; ++l) {
     h->len[l] = 0;
     h->pending[l] = 0;
@@ -683,6 +786,7 @@ regmem_status regmem_export_bank(regmem_t* h, int32_t layer, void* hostK, void* 
   if (n == 0) return REGMEM_OK;
   const size_t row = kHeadDim * 2;
   const size_t off = (size_t)layer * h->heads * h->cap * kHeadDim;
+  if ((s = join_side(h)) != REGMEM_OK) return s;  // admissions still appending on the side stream
   RM_CUDA(h, cudaMemcpy2DAsync(hostK, n * row, h->bankK + off, h->cap * row, n * row, h->heads,
                                cudaMemcpyDeviceToHost, h->stream));
   RM_CUDA(h, cudaMemcpy2DAsync(hostV, n * row, h->bankV + off, h->cap * row, n * row, h->heads,
@@ -700,6 +804,7 @@ regmem_status regmem_import_bank(regmem_t* h, int32_t layer, const void* hostK, 
   if (len > 0 && (!hostK || !hostV)) return fail(h, REGMEM_ERR_ARG, "null host pointer");
   const size_t row = kHeadDim * 2;
   const size_t off = (size_t)layer * h->heads * h->cap * kHeadDim;
+  if ((s = join_side(h)) != REGMEM_OK) return s;
   if (len > 0) {
     RM_CUDA(h, cudaMemcpy2DAsync(h->bankK + off, h->cap * row, hostK, len * row, len * row,
                                  h->heads, cudaMemcpyHostToDevice, h->stream));
@@ -716,7 +821,7 @@ regmem_status regmem_copy_lse(regmem_t* h, float* dst) {
   regmem_status s = ready(h, 0, false);
   if (s != REGMEM_OK) return s;
   if (!dst) return fail(h, REGMEM_ERR_ARG, "null pointer");
-  RM_CUDA(h, cudaMemcpyAsync(dst, h->lse, (size_t)h->heads * h->N * sizeof(float),
+  RM_CUDA(h, cudaMemcpyAsync(dst, lse_of(h, h->lse_layer), (size_t)h->heads * h->N * sizeof(float),
                              cudaMemcpyDeviceToDevice, h->stream));
   return REGMEM_OK;
 }
@@ -727,6 +832,7 @@ regmem_status regmem_synchronize(regmem_t* h) {
     if (cudaSetDevice(h->device) != cudaSuccess)
       return fail(h, REGMEM_ERR_CUDA, "cannot select device %d", h->device);
     RM_CUDA(h, cudaStreamSynchronize(h->stream));
+    if (h->sstream) RM_CUDA(h, cudaStreamSynchronize(h->sstream));
     if (h->cstream) RM_CUDA(h, cudaStreamSynchronize(h->cstream));
     if (h->dstream) RM_CUDA(h, cudaStreamSynchronize(h->dstream));
     RM_CUDA(h, cudaGetLastError());
@@ -766,6 +872,7 @@ void regmem_destroy(regmem_t* h) {
   if (h->frame_set) {
     cudaSetDevice(h->device);
     cudaStreamSynchronize(h->stream);
+    if (h->sstream) cudaStreamSynchronize(h->sstream);
     if (h->cstream) cudaStreamSynchronize(h->cstream);
     if (h->dstream) cudaStreamSynchronize(h->dstream);
   }
@@ -796,6 +903,9 @@ void regmem_destroy(regmem_t* h) {
   }
   if (h->cstream) cudaStreamDestroy(h->cstream);
   if (h->dstream) cudaStreamDestroy(h->dstream);
+  if (h->sstream) cudaStreamDestroy(h->sstream);
+  if (h->main_ev) cudaEventDestroy(h->main_ev);
+  if (h->side_ev) cudaEventDestroy(h->side_ev);
   delete h;
 }
 

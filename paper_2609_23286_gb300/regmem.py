@@ -23,6 +23,8 @@ _SIGNATURES = {
     "regmem_create": (ctypes.c_int, [ctypes.POINTER(_P), _I32, _I32, _I32, _I32]),
     "regmem_set_frame": (ctypes.c_int, [_P, _P]),
     "regmem_set_stream": (ctypes.c_int, [_P, _P]),
+    "regmem_set_overlap": (ctypes.c_int, [_P, _I32]),
+    "regmem_join": (ctypes.c_int, [_P]),
     "regmem_attend_frame": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P]),
     "regmem_attend_frame_host": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P]),
     "regmem_admit": (ctypes.c_int, [_P, _I32, _I32, _P]),
@@ -138,6 +140,14 @@ def regmem_set_frame(h, n_tokens, n_special, grid_h, grid_w, ds=2, max_frames=1,
 
 def regmem_set_stream(h, stream):
     return _check(h, load().regmem_set_stream(h, _stream_ptr(stream)))
+
+
+def regmem_set_overlap(h, on):
+    return _check(h, load().regmem_set_overlap(h, int(on)))
+
+
+def regmem_join(h):
+    return _check(h, load().regmem_join(h))
 
 
 def _stream_ptr(stream):
@@ -260,6 +270,12 @@ class RegMem:
 
     def set_stream(self, stream):
         return regmem_set_stream(self.h, stream)
+
+    def set_overlap(self, on):
+        return regmem_set_overlap(self.h, on)
+
+    def join(self):
+        return regmem_join(self.h)
 
     def attend_frame(self, layer, Q, K, V, out, saliency):
         return regmem_attend_frame(self.h, layer, Q, K, V, out, saliency)

@@ -66,6 +66,12 @@ def test_host_side_validation_without_gpu(lib_path):
         fd = regmem.FrameDesc(70, 5, 8, 8, 2, 4, 0.0, 0)      # 70 != 5 + 64
         assert lib.regmem_set_frame(handle, ctypes.byref(fd)) == regmem.ERR_ARG
         assert lib.regmem_reset(handle) == 0
+        assert lib.regmem_set_overlap(handle, 2) == regmem.ERR_ARG
+        assert lib.regmem_set_overlap(handle, 1) == 0      # takes effect at the first attend
+        assert lib.regmem_join(handle) == 0                 # no side work yet
+        assert lib.regmem_set_overlap(handle, 0) == 0
     finally:
         regmem.regmem_destroy(handle)
     assert lib.regmem_reset(None) == regmem.ERR_ARG
+    assert lib.regmem_set_overlap(None, 1) == regmem.ERR_ARG
+    assert lib.regmem_join(None) == regmem.ERR_ARG

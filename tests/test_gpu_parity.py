@@ -385,6 +385,114 @@ def test_fused_step_matches_two_calls():
         b.close()
 
 
+def _enqueue_stream(st, frames, ks, high_priority=False):
+    """Enqueue every (frame, layer) step of st back to back, without host
+    synchronisation, each into buffers of its own; returns them after a
+    device synchronisation.  ks[layer] rows are admitted per frame."""
+    stream = (torch.cuda.Stream(priority=-1) if high_priority else torch.cuda.current_stream())
+    torch.cuda.synchronize()
+    st.rm.set_stream(stream)
+    res = []
+    inputs = [[st.inputs(layer, t) for layer in range(st.L)] for t in range(1, frames + 1)]
+    torch.cuda.synchronize()
+    for t in range(frames):
+        for layer in range(st.L):
+            q, kk, v = inputs[t][layer]
+            out = torch.empty_like(q)
+            sal = torch.empty(st.H, st.N, dtype=torch.float32, device="cuda")
+            lse = torch.empty(st.H, st.N, dtype=torch.float32, device="cuda")
+            idx = torch.full((st.H, max(ks[layer], 1)), -1, dtype=torch.int32, device="cuda")
+            st.rm.attend_admit(layer, q, kk, v, out, sal, ks[layer], idx)
+            st.rm.copy_lse(lse)
+            res.append((out, sal, lse, idx))
+    st.rm.join()
+    torch.cuda.synchronize()
+    st.rm.synchronize()
+    return res, inputs
+
+
+@pytest.mark.parametrize("ks", [(14, 14, 14), (14, 40, 1)])
+def test_overlap_matches_one_stream(ks):
+    """regmem_set_overlap(1): saliency and admission on the side stream,
+    every step enqueued back to back (so side work of layer l runs beside the
+    attention of layer l + 1 and the next frame's attention must wait for
+    it), on a high-priority stream.  Outputs, LSE, saliency, indices and
+    banks equal the one-stream run bit for bit; k = 40 takes the separate
+    selection kernel on the side stream, k = 1 the fused one."""
+    H, ns, gh, gw = 16, 5, 37, 37
+    frames = 5
+    a = Stream(3, H, ns, gh, gw, budget=max(ks), max_frames=frames, seed=31)
+    b = Stream(3, H, ns, gh, gw, budget=max(ks), max_frames=frames, seed=31)
+    try:
+        b.rm.set_overlap(1)
+        ra, _ = _enqueue_stream(a, frames, ks)
+        rb, _ = _enqueue_stream(b, frames, ks, high_priority=True)
+        for i, (x, y) in enumerate(zip(ra, rb)):
+            t, layer = divmod(i, 3)
+            for name, u, w in zip(("out", "saliency", "lse", "idx"), x, y):
+                if name == "idx" and t == 0:
+                    continue  # the first frame is stored whole: no indices
+                assert torch.equal(u, w), f"{name} differs at t={t + 1} layer={layer}"
+        for layer in range(3):
+            assert a.rm.memory_len(layer) == b.rm.memory_len(layer)
+            ka, va = a.export(layer)
+            kb, vb = b.export(layer)
+            assert torch.equal(ka, kb) and torch.equal(va, vb)
+    finally:
+        a.close()
+        b.close()
+
+
+def test_overlap_against_oracle_and_mode_switches():
+    """Overlap on a 2-layer 13 x 11 + 5 stream checked against the oracle
+    frame by frame; then the two-call path, the host-buffer path, an import
+    and a reset on the same handle, each ordered after pending side work."""
+    H, ns, gh, gw, k = 4, 5, 13, 11, 3
+    st = Stream(2, H, ns, gh, gw, budget=k, max_frames=8, seed=32)
+    ref = orc.OracleStream(2, H, 64, ns, gh, gw)
+    try:
+        st.rm.set_overlap(1)
+        for t in range(1, 5):
+            for layer in range(2):
+                q, kk, v = st.inputs(layer, t)
+                if t == 3 and layer == 1:   # two-call path between overlapped steps
+                    out, sal, lse = st.attend(layer, q, kk, v)
+                    idx = st.admit(layer, k)
+                else:
+                    out, sal, lse, idx = st.attend_admit(layer, q, kk, v, k)
+                torch.cuda.synchronize()
+                r = ref.attend(layer, to64(q), to64(kk), to64(v))
+                check_o(out, r["O"], f"t={t} l={layer}")
+                check_lse(lse, r["LSE"], f"t={t} l={layer}")
+                check_saliency(sal, r["S"], f"t={t} l={layer}")
+                if t == 1:
+                    ref.admit(layer, k)
+                else:
+                    gi = idx.cpu().numpy().astype(np.int64)
+                    check_indices(gi, to64(sal), r["S"], ns, k, len(ref.qidx))
+                    ref.admit(layer, k, indices=gi)
+        # host-buffer path with overlap: same outputs as the device path
+        q, kk, v = st.inputs(0, 5)
+        hq, hk, hv = q.cpu().pin_memory(), kk.cpu().pin_memory(), v.cpu().pin_memory()
+        ho = torch.empty_like(hq).pin_memory()
+        hs = torch.empty(H, st.N, dtype=torch.float32).pin_memory()
+        st.rm.attend_admit_host(0, hq, hk, hv, ho, hs, k)
+        st.rm.synchronize()
+        r = ref.attend(0, to64(q), to64(kk), to64(v))
+        check_o(ho, r["O"], "host path")
+        check_saliency(hs, r["S"], "host path")
+        # import and export follow the pending side work
+        bk, bv = st.export(1)
+        st.rm.import_bank(1, bk, bv, bk.shape[1])
+        bk2, bv2 = st.export(1)
+        assert torch.equal(bk, bk2) and torch.equal(bv, bv2)
+        st.rm.reset()
+        st.rm.set_overlap(0)
+        assert st.rm.memory_len(0) == 0
+    finally:
+        st.close()
+
+
 def test_fused_uniform_keys_and_every_candidate():
     """The fused selection: uniform saliency ties to the lowest indices, and
     k = all candidates admits every patch token in order."""
