@@ -278,7 +278,11 @@ REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_frame_desc* fd
  * recorded on the handle's stream immediately before and after the sampled
  * launches of the attention kernel and after the merge of split units that
  * follows it: attention_ms sums the attention kernel's intervals, merge_ms
- * the merge's; the other kernels are not bracketed. */
+ * the merge's; the other kernels are not bracketed.  It also turns on the
+ * attention kernel's own launch clock for EVERY attention launch: the GPU's
+ * global timer from the first CTA past the launch's dependency wait to the
+ * last CTA's end, summed in device memory (no event between launches, so it
+ * does not perturb the stream it measures). */
 typedef struct regmem_profile {
   int64_t launches_attention; /* attention kernel (attend and frame attention)  */
   int64_t launches_saliency;  /* LSE-saliency kernel                            */
@@ -295,6 +299,9 @@ typedef struct regmem_profile {
   int32_t attention_ctas_per_sm; /* resident attention CTAs per SM (occupancy) */
   double merge_ms;            /* summed event time of the merges of split units
                                  behind those launches                          */
+  int64_t attention_clocked;  /* attention launches measured by the launch clock */
+  double attention_clock_ms;  /* their summed durations (global timer)          */
+  double attention_clock_flops; /* algorithmic FLOPs of those launches          */
 } regmem_profile;
 
 /* Resets the counters; time_attention = n >= 1 also brackets every n-th

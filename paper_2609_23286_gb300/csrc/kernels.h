@@ -65,6 +65,10 @@ struct AttnArgs {
   float* part_lse;          // [grid][2][kUnitRows]
   int* status;
   int grid;                 // CTAs of the attention kernel (<= plan.total)
+  // optional launch clock (nullptr: off), 5 words: [0] earliest CTA start
+  // after the dependency wait (~0 when idle), [1] CTAs finished, [2] sum of
+  // launch durations in ns, [3] launches summed, [4] latest CTA end
+  unsigned long long* clk;
 };
 
 // Work decomposition: a unit is (head, pair of 128-row query tiles); each

@@ -45,6 +45,7 @@ struct regmem {
   __nv_bfloat16* part_o = nullptr;  // split-KV partials
   float* part_lse = nullptr;
   int* head_done = nullptr;   // per-head completion counters of the distributed selection
+  unsigned long long* kclock = nullptr;  // the attention's launch clock (AttnArgs::clk)
   uint64_t* adm_lists = nullptr;  // per-(head, key tile) candidate lists, [H][nkt][32]
   int attn_grid = 0;
   int attn_ctas_per_sm = 0;
@@ -242,6 +243,7 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   a.part_o = h->part_o;
   a.part_lse = h->part_lse;
   a.status = h->status_dev;
+  a.clk = h->time_every > 0 ? h->kclock : nullptr;
   const AttnPlan pl = attn_plan(h->N, h->heads, M);
   const long long G = pl.total < h->attn_grid ? pl.total : h->attn_grid;
   a.grid = (int)G;
@@ -268,6 +270,7 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   const double L = (double)M + h->N;
   h->prof.launches_attention += 1;
   if (a.grid > 1) h->prof.launches_combine += 1;
+  if (a.clk) h->prof.attention_clock_flops += 4.0 * h->N * L * kHeadDim * h->heads;
   if (timed) {
     h->prof.attention_timed += 1;
     h->prof.attention_flops += 4.0 * h->N * L * kHeadDim * h->heads;
@@ -363,6 +366,9 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
   RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_elems(h->attn_grid) * sizeof(__nv_bfloat16)));
   RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid) * sizeof(float)));
+  RM_CUDA(h, cudaMalloc(&h->kclock, 5 * sizeof(unsigned long long)));
+  RM_CUDA(h, cudaMemset(h->kclock, 0xFF, sizeof(unsigned long long)));
+  RM_CUDA(h, cudaMemset(h->kclock + 1, 0, 4 * sizeof(unsigned long long)));
   RM_CUDA(h, cudaMalloc(&h->head_done, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMemset(h->head_done, 0, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMalloc(&h->adm_lists, (size_t)h->heads * ((N + kTile - 1) / kTile) * 32 * sizeof(uint64_t)));
@@ -850,6 +856,10 @@ regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention) {
   }
   h->prof = regmem_profile{};
   h->time_every = time_attention > 0 ? time_attention : 0;
+  if (h->frame_set) {  // restart the launch clock (stream-ordered after earlier launches)
+    RM_CUDA(h, cudaMemsetAsync(h->kclock, 0xFF, sizeof(unsigned long long), h->stream));
+    RM_CUDA(h, cudaMemsetAsync(h->kclock + 1, 0, 4 * sizeof(unsigned long long), h->stream));
+  }
   h->attn_launch_no = 0;
   return REGMEM_OK;
 }
@@ -862,6 +872,10 @@ regmem_status regmem_profile_read(regmem_t* h, regmem_profile* out) {
     RM_CUDA(h, cudaStreamSynchronize(h->stream));
     for (size_t i = 0; i < h->ev_busy.size(); ++i)
       if (h->ev_busy[i]) RM_CUDA(h, harvest_pair(h, i));
+    unsigned long long w[5];
+    RM_CUDA(h, cudaMemcpy(w, h->kclock, sizeof(w), cudaMemcpyDeviceToHost));
+    h->prof.attention_clocked = (int64_t)w[3];
+    h->prof.attention_clock_ms = (double)w[2] * 1e-6;
   }
   *out = h->prof;
   return check_device_status(h);
@@ -883,6 +897,7 @@ void regmem_destroy(regmem_t* h) {
   cudaFree(h->part_o);
   cudaFree(h->part_lse);
   cudaFree(h->head_done);
+  cudaFree(h->kclock);
   cudaFree(h->adm_lists);
   if (h->status_host) cudaFreeHost(h->status_host);
   cudaFree(h->stQ);
