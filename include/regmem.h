@@ -281,8 +281,11 @@ REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_frame_desc* fd
  * the merge's; the other kernels are not bracketed.  It also turns on the
  * attention kernel's own launch clock for EVERY attention launch: the GPU's
  * global timer from the first CTA past the launch's dependency wait to the
- * last CTA's end, summed in device memory (no event between launches, so it
- * does not perturb the stream it measures). */
+ * last CTA's end, kept per launch in 16 MB of device memory (allocated by
+ * the first regmem_profile_enable after regmem_set_frame) for up to 2^20
+ * launches per profiling window, and summed by regmem_profile_read.  No
+ * event sits between launches, so it does not perturb the stream it
+ * measures. */
 typedef struct regmem_profile {
   int64_t launches_attention; /* attention kernel (attend and frame attention)  */
   int64_t launches_saliency;  /* LSE-saliency kernel                            */

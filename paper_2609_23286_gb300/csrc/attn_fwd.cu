@@ -121,7 +121,8 @@ struct Params {
   __nv_bfloat16* part_o;  // [grid][2][256][64]: partials of each CTA's first / last piece
   float* part_lse;  // [grid][2][256]
   int* status;
-  unsigned long long* clk;  // launch clock (AttnArgs::clk) or nullptr
+  unsigned long long* clk_start;  // launch clock (AttnArgs) or nullptr
+  unsigned long long* clk_end;
 };
 
 using split::cta_of;
@@ -192,7 +193,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   grid_dep_wait();  // the previous kernel's writes are visible, its reads done
-  if (p.clk && tid == 0) atomicMin(&p.clk[0], globaltimer_ns());
+  if (p.clk_start && tid == 0) atomicMin(p.clk_start, globaltimer_ns());
 
   if (warp < 4) {
    setmaxnreg_dec<REGS_CTRL>();
@@ -533,21 +534,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     tmem_dealloc(tmem, TMEM_COLS);
   }
   if (tid == 0 && sm.abort_flag) atomicOr(p.status, kStatusTimeout);
-  if (p.clk && tid == 0) {
-    // launch clock: the last CTA to finish adds (latest end - earliest start)
-    // and resets the start and end words for the next launch, which reads
-    // them only after its own dependency wait, i.e. after this kernel
-    atomicMax(&p.clk[4], globaltimer_ns());
-    __threadfence();
-    if (atomicAdd(&p.clk[1], 1ull) == (unsigned long long)(G - 1)) {
-      __threadfence();
-      const unsigned long long t1 = atomicExch(&p.clk[4], 0ull);
-      const unsigned long long t0 = atomicExch(&p.clk[0], ~0ull);
-      atomicExch(&p.clk[1], 0ull);
-      atomicAdd(&p.clk[2], t1 - t0);
-      atomicAdd(&p.clk[3], 1ull);
-    }
-  }
+  // launch clock: fire-and-forget reductions, nothing waits for them
+  if (p.clk_end && tid == 0) atomicMax(p.clk_end, globaltimer_ns());
   // The merge kernel behind is released only as CTAs finish: released at the
   // start, its small blocks took SMs as they freed up and held them while
   // waiting, which measured 25 us slower per launch.
@@ -583,7 +571,8 @@ Params make_params(const AttnArgs& a) {
   p.part_o = a.part_o;
   p.part_lse = a.part_lse;
   p.status = a.status;
-  p.clk = a.clk;
+  p.clk_start = a.clk_start;
+  p.clk_end = a.clk_end;
   return p;
 }
 

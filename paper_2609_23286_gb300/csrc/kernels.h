@@ -65,10 +65,11 @@ struct AttnArgs {
   float* part_lse;          // [grid][2][kUnitRows]
   int* status;
   int grid;                 // CTAs of the attention kernel (<= plan.total)
-  // optional launch clock (nullptr: off), 5 words: [0] earliest CTA start
-  // after the dependency wait (~0 when idle), [1] CTAs finished, [2] sum of
-  // launch durations in ns, [3] launches summed, [4] latest CTA end
-  unsigned long long* clk;
+  // optional launch clock (nullptr: off), this launch's words, global timer
+  // in ns: the earliest CTA start after the dependency wait (preset to ~0)
+  // and the latest CTA end (preset to 0)
+  unsigned long long* clk_start;
+  unsigned long long* clk_end;
 };
 
 // Work decomposition: a unit is (head, pair of 128-row query tiles); each

@@ -45,7 +45,10 @@ struct regmem {
   __nv_bfloat16* part_o = nullptr;  // split-KV partials
   float* part_lse = nullptr;
   int* head_done = nullptr;   // per-head completion counters of the distributed selection
-  unsigned long long* kclock = nullptr;  // the attention's launch clock (AttnArgs::clk)
+  // the attention's launch clock: kClockSlots start words, then as many end
+  // words, one pair per launch since regmem_profile_enable
+  unsigned long long* kclock = nullptr;
+  long long clk_next = 0;
   uint64_t* adm_lists = nullptr;  // per-(head, key tile) candidate lists, [H][nkt][32]
   int attn_grid = 0;
   int attn_ctas_per_sm = 0;
@@ -186,6 +189,7 @@ regmem_status ready(regmem_t* h, int layer, bool need_layer) {
 }
 
 constexpr size_t kEventPairs = 256;
+constexpr long long kClockSlots = 1 << 20;  // launches one profiling window can clock (16 MB)
 
 // Adds the elapsed times of event triple i to the profile and frees the slot.
 cudaError_t harvest_pair(regmem_t* h, size_t i) {
@@ -243,7 +247,11 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   a.part_o = h->part_o;
   a.part_lse = h->part_lse;
   a.status = h->status_dev;
-  a.clk = h->time_every > 0 ? h->kclock : nullptr;
+  if (h->kclock && h->time_every > 0 && h->clk_next < kClockSlots) {
+    a.clk_start = h->kclock + h->clk_next;
+    a.clk_end = h->kclock + kClockSlots + h->clk_next;
+    ++h->clk_next;
+  }
   const AttnPlan pl = attn_plan(h->N, h->heads, M);
   const long long G = pl.total < h->attn_grid ? pl.total : h->attn_grid;
   a.grid = (int)G;
@@ -270,7 +278,7 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   const double L = (double)M + h->N;
   h->prof.launches_attention += 1;
   if (a.grid > 1) h->prof.launches_combine += 1;
-  if (a.clk) h->prof.attention_clock_flops += 4.0 * h->N * L * kHeadDim * h->heads;
+  if (a.clk_start) h->prof.attention_clock_flops += 4.0 * h->N * L * kHeadDim * h->heads;
   if (timed) {
     h->prof.attention_timed += 1;
     h->prof.attention_flops += 4.0 * h->N * L * kHeadDim * h->heads;
@@ -366,9 +374,6 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
   RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_elems(h->attn_grid) * sizeof(__nv_bfloat16)));
   RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid) * sizeof(float)));
-  RM_CUDA(h, cudaMalloc(&h->kclock, 5 * sizeof(unsigned long long)));
-  RM_CUDA(h, cudaMemset(h->kclock, 0xFF, sizeof(unsigned long long)));
-  RM_CUDA(h, cudaMemset(h->kclock + 1, 0, 4 * sizeof(unsigned long long)));
   RM_CUDA(h, cudaMalloc(&h->head_done, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMemset(h->head_done, 0, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMalloc(&h->adm_lists, (size_t)h->heads * ((N + kTile - 1) / kTile) * 32 * sizeof(uint64_t)));
@@ -856,9 +861,12 @@ regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention) {
   }
   h->prof = regmem_profile{};
   h->time_every = time_attention > 0 ? time_attention : 0;
-  if (h->frame_set) {  // restart the launch clock (stream-ordered after earlier launches)
-    RM_CUDA(h, cudaMemsetAsync(h->kclock, 0xFF, sizeof(unsigned long long), h->stream));
-    RM_CUDA(h, cudaMemsetAsync(h->kclock + 1, 0, 4 * sizeof(unsigned long long), h->stream));
+  h->clk_next = 0;
+  if (h->frame_set && h->time_every > 0) {  // preset the slots, stream-ordered before the launches
+    const size_t bytes = 2 * kClockSlots * sizeof(unsigned long long);
+    if (!h->kclock) RM_CUDA(h, cudaMalloc(&h->kclock, bytes));
+    RM_CUDA(h, cudaMemsetAsync(h->kclock, 0xFF, bytes / 2, h->stream));
+    RM_CUDA(h, cudaMemsetAsync(h->kclock + kClockSlots, 0, bytes / 2, h->stream));
   }
   h->attn_launch_no = 0;
   return REGMEM_OK;
@@ -872,10 +880,19 @@ regmem_status regmem_profile_read(regmem_t* h, regmem_profile* out) {
     RM_CUDA(h, cudaStreamSynchronize(h->stream));
     for (size_t i = 0; i < h->ev_busy.size(); ++i)
       if (h->ev_busy[i]) RM_CUDA(h, harvest_pair(h, i));
-    unsigned long long w[5];
-    RM_CUDA(h, cudaMemcpy(w, h->kclock, sizeof(w), cudaMemcpyDeviceToHost));
-    h->prof.attention_clocked = (int64_t)w[3];
-    h->prof.attention_clock_ms = (double)w[2] * 1e-6;
+    if (h->kclock && h->clk_next > 0) {
+      const size_t n = (size_t)h->clk_next;
+      std::vector<unsigned long long> t0(n), t1(n);
+      RM_CUDA(h, cudaMemcpy(t0.data(), h->kclock, n * sizeof(unsigned long long),
+                            cudaMemcpyDeviceToHost));
+      RM_CUDA(h, cudaMemcpy(t1.data(), h->kclock + kClockSlots, n * sizeof(unsigned long long),
+                            cudaMemcpyDeviceToHost));
+      double ns = 0.0;
+      for (size_t i = 0; i < n; ++i)
+        if (t1[i] > t0[i]) ns += (double)(t1[i] - t0[i]);
+      h->prof.attention_clocked = h->clk_next;
+      h->prof.attention_clock_ms = ns * 1e-6;
+    }
   }
   *out = h->prof;
   return check_device_status(h);
