@@ -75,3 +75,24 @@ def test_host_side_validation_without_gpu(lib_path):
     assert lib.regmem_reset(None) == regmem.ERR_ARG
     assert lib.regmem_set_overlap(None, 1) == regmem.ERR_ARG
     assert lib.regmem_join(None) == regmem.ERR_ARG
+
+
+def _c_struct_fields(name):
+    """(type, field) pairs of a typedef struct in the header, in order."""
+    src = open(HEADER).read()
+    body = re.search(r"typedef struct %s \{(.*?)\} %s;" % (name, name), src, re.S).group(1)
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    return re.findall(r"\b(int32_t|int64_t|double|float)\s+(\w+)\s*;", body)
+
+
+@pytest.mark.parametrize("cname, pyname", [("regmem_profile", "Profile"),
+                                           ("regmem_frame_desc", "FrameDesc")])
+def test_binding_structs_match_header(cname, pyname):
+    """The ctypes mirrors of the header's structs have the same fields, in the
+    same order, with the same C types (a mismatch would read garbage)."""
+    from paper_2609_23286_gb300 import regmem
+    ctype = {"int32_t": ctypes.c_int32, "int64_t": ctypes.c_int64, "double": ctypes.c_double,
+             "float": ctypes.c_float}
+    want = [(f, ctype[t]) for t, f in _c_struct_fields(cname)]
+    got = [(f, t) for f, t in getattr(regmem, pyname)._fields_]
+    assert got == want

@@ -584,3 +584,39 @@ def test_selection_on_crafted_saliency(pattern, k):
             assert list(idx[h].cpu().numpy()) == orc.topk_admission(c[h], ns, k), f"head {h}"
     finally:
         st.close()
+
+
+def test_profile_counters_events_and_launch_clock():
+    """regmem_profile_*: launch counters, event timing of every launch
+    (time_attention = 1) and the attention's launch clock agree with each
+    other; with profiling off nothing is timed."""
+    H, ns, gh, gw, k = 16, 5, 37, 37, 14
+    st = Stream(2, H, ns, gh, gw, budget=k, max_frames=6, seed=33)
+    try:
+        st.rm.set_overlap(1)
+        for layer in range(2):
+            st.attend_admit(layer, *st.inputs(layer, 1), k)
+        st.rm.profile_enable(1)
+        for t in (2, 3, 4):
+            for layer in range(2):
+                st.attend_admit(layer, *st.inputs(layer, t), k)
+        p = st.rm.profile_read()
+        assert p.launches_attention == 6 and p.launches_saliency == 6
+        assert p.launches_combine == (6 if p.attention_ctas > 1 else 0)
+        assert p.attention_timed == 6 and p.attention_clocked == 6
+        assert p.attention_clock_flops == pytest.approx(p.attention_flops, rel=1e-12)
+        L = [ns + gh * gw + (ns + gh * gw) + (t - 2) * k for t in (2, 3, 4)]
+        assert p.attention_flops == pytest.approx(sum(4.0 * (ns + gh * gw) * l * 64 * H * 2 for l in L))
+        # the clock brackets the kernel after its dependency wait; the events
+        # also hold its launch: clock <= events, and of the same order
+        assert 0 < p.attention_clock_ms <= 1.05 * p.attention_ms + 0.005
+        assert p.attention_clock_ms >= 0.3 * p.attention_ms
+        st.rm.profile_enable(0)
+        for layer in range(2):
+            st.attend_admit(layer, *st.inputs(layer, 5), k)
+        p = st.rm.profile_read()
+        assert p.launches_attention == 2 and p.attention_timed == 0 and p.attention_clocked == 0
+        assert p.attention_clock_ms == 0.0
+        st.rm.synchronize()
+    finally:
+        st.close()
