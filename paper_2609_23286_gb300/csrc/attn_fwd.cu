@@ -9,8 +9,10 @@
 // into 128-row tiles: ceil(M/128) bank tiles followed by ceil(N/128) frame
 // tiles, each possibly ragged (columns past the valid count are masked).
 //
-// Work split (stream-K over the key dimension): a unit is (head, pair of
-// consecutive 128-row query tiles); the (unit, key tile) space is cut into
+// Work split (stream-K over the key dimension): a unit is a pair of 128-row
+// query tiles -- two consecutive tiles of one head, or the last tiles of two
+// heads when a head has an odd number of them (unit_tiles) -- and the
+// (unit, key tile) space is cut into
 // `grid` contiguous equal ranges, one per CTA (one CTA per SM).  A unit whose
 // key tiles all fall in one CTA is finished there (O in bf16 and LSE written
 // directly).  A unit cut between CTAs leaves one normalised fp32 partial
@@ -25,8 +27,9 @@
 //
 // CTA layout, warp-specialised (12 warps, three warpgroups):
 //   warp 0       TMA producer: both Q tiles of a unit, then K and V tiles
-//                through a 5-stage ring (a stage holds one K and one V tile,
-//                which land on one barrier)
+//                through a 6-stage ring (a stage holds one K and one V tile,
+//                which land on one barrier; a two-head unit takes two stages
+//                per key tile, one per head)
 //   warp 1       Q K^T issuer (one lane) for both query tiles; owns TMEM
 //   warps 2, 3   P V issuers (one lane each) for query tile 0 and 1
 // The control warpgroup (warps 0-3) hands most of its register budget to
@@ -34,7 +37,9 @@
 //   warps 4..7   softmax warpgroup 0 -> query tile 0 of the unit
 //   warps 8..11  softmax warpgroup 1 -> query tile 1 of the unit
 // Each softmax thread owns one query row (its TMEM lane).  Each key tile is
-// loaded once and serves both query tiles.
+// loaded once and serves both query tiles (once per head for a two-head
+// unit: each tile reads its own head's stage, and the other tile's P V
+// issuer releases that stage with a plain arrival).
 // TMEM (512 columns): S0 [0,128), S1 [128,256) fp32 logits; P0 [256,320),
 // P1 [320,384) bf16 probabilities packed two per column; O0 [384,448),
 // O1 [448,512) fp32 accumulators.  Q K^T is an SS-MMA (Q, K K-major in smem);
@@ -75,7 +80,7 @@ namespace {
 
 constexpr int BM = kTile, BN = kTile, HD = kHeadDim;
 constexpr int UROWS = kUnitRows;         // query rows per unit (two tiles)
-constexpr int STAGES = 5;  // K/V ring depth (a stage holds one K tile and one V tile)
+constexpr int STAGES = 6;  // K/V ring depth (a stage holds one K tile and one V tile)
 constexpr int TILE_BYTES = BM * HD * 2;  // 16 KB bf16 tile
 constexpr int THREADS = 384;
 // Register split: launched at 168 per thread (384 x 168 = 64,512); the
@@ -110,10 +115,11 @@ struct Smem {
 // The dynamic shared window is requested 1 KB aligned (128-byte swizzle
 // atoms need it) and checked at run time.
 constexpr size_t SMEM_BYTES = (sizeof(Smem) + 127) & ~size_t(127);
+static_assert(SMEM_BYTES <= 232448, "more dynamic shared memory than a CTA can have (227 KB)");
 
 struct Params {
   int N, H, M;
-  int nb, nkv, nqt, nqp;
+  int nb, nkv, nqt;
   long long total;
   float scale_log2;
   __nv_bfloat16* out;
@@ -134,17 +140,17 @@ __device__ __forceinline__ int tile_valid(const Params& p, int j) {
 
 // One piece of a CTA's range: unit u, key tiles [j0, j1).
 struct Piece {
-  int u, j0, j1, h, qp;
-  bool has1;  // the unit's second query tile holds rows
+  int u, j0, j1;
+  UnitTiles ut;  // the unit's two query tiles (head, tile index)
+  int kvs;       // K/V stages per key tile: 2 when the tiles belong to two heads
 };
 __device__ __forceinline__ Piece piece_at(const Params& p, long long x, long long x_end) {
   Piece pc;
   pc.u = (int)(x / p.nkv);
   pc.j0 = (int)(x - (long long)pc.u * p.nkv);
   pc.j1 = (int)min((long long)p.nkv, pc.j0 + (x_end - x));
-  pc.h = pc.u / p.nqp;
-  pc.qp = pc.u - pc.h * p.nqp;
-  pc.has1 = 2 * pc.qp + 1 < p.nqt;
+  pc.ut = unit_tiles(pc.u, p.nqt, p.H);
+  pc.kvs = pc.ut.h0 != pc.ut.h1 ? 2 : 1;
   return pc;
 }
 
@@ -213,25 +219,28 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (!ok) break;
         const uint32_t bq = smem_addr(&sm.q_full);
         mbar_arrive_expect_tx(bq, 2 * TILE_BYTES);
-        tma_load_3d(smem_addr(sm.q[0]), &tmQ, bq, 0, pc.h, (2 * pc.qp) * BM);
-        tma_load_3d(smem_addr(sm.q[1]), &tmQ, bq, 0, pc.h, (2 * pc.qp + 1) * BM);
+        // (a unit without a second tile loads rows past the frame: zero fill)
+        tma_load_3d(smem_addr(sm.q[0]), &tmQ, bq, 0, pc.ut.h0, pc.ut.qt0 * BM);
+        tma_load_3d(smem_addr(sm.q[1]), &tmQ, bq, 0, pc.ut.h1, pc.ut.qt1 * BM);
         ++piece;
         for (int j = pc.j0; j < pc.j1 && ok; ++j) {
-          const int st = nkv % STAGES;
-          if (nkv >= STAGES)
-            ok = mbar_wait(smem_addr(&sm.kv_empty[st]), ((nkv / STAGES) - 1) & 1, abort_flag, WAIT_NS);
-          if (!ok) break;
-          // K and V of the tile land on one barrier: the issuer waits once
-          const uint32_t bkv = smem_addr(&sm.kv_full[st]);
-          mbar_arrive_expect_tx(bkv, 2 * TILE_BYTES);
-          if (j < p.nb) {
-            tma_load_3d(smem_addr(sm.k[st]), &tmBK, bkv, 0, j * BN, pc.h);
-            tma_load_3d(smem_addr(sm.v[st]), &tmBV, bkv, 0, j * BN, pc.h);
-          } else {
-            tma_load_3d(smem_addr(sm.k[st]), &tmK, bkv, 0, pc.h, (j - p.nb) * BN);
-            tma_load_3d(smem_addr(sm.v[st]), &tmV, bkv, 0, pc.h, (j - p.nb) * BN);
+          for (int hs = 0; hs < pc.kvs && ok; ++hs) {  // one stage per head of the unit
+            const int st = nkv % STAGES, h = hs ? pc.ut.h1 : pc.ut.h0;
+            if (nkv >= STAGES)
+              ok = mbar_wait(smem_addr(&sm.kv_empty[st]), ((nkv / STAGES) - 1) & 1, abort_flag, WAIT_NS);
+            if (!ok) break;
+            // K and V of the tile land on one barrier: the issuer waits once
+            const uint32_t bkv = smem_addr(&sm.kv_full[st]);
+            mbar_arrive_expect_tx(bkv, 2 * TILE_BYTES);
+            if (j < p.nb) {
+              tma_load_3d(smem_addr(sm.k[st]), &tmBK, bkv, 0, j * BN, h);
+              tma_load_3d(smem_addr(sm.v[st]), &tmBV, bkv, 0, j * BN, h);
+            } else {
+              tma_load_3d(smem_addr(sm.k[st]), &tmK, bkv, 0, h, (j - p.nb) * BN);
+              tma_load_3d(smem_addr(sm.v[st]), &tmV, bkv, 0, h, (j - p.nb) * BN);
+            }
+            ++nkv;
           }
-          ++nkv;
         }
         x += pc.j1 - pc.j0;
       }
@@ -258,19 +267,24 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int n = pc.j1 - pc.j0;
         x += n;
         ++piece;
-        const int ntiles = pc.has1 ? 2 : 1;  // query tiles of this unit
-        const int t0 = it;  // CTA-local index of the piece's first key tile
-        it += n;
+        const int ntiles = pc.ut.has1 ? 2 : 1;  // query tiles of this unit
+        // CTA-local stage use of key tile jj for query tile t: one stage per
+        // key tile, or two (one per head) when the tiles belong to two heads
+        const int t0 = it;
+        it += n * pc.kvs;
+        auto use_of = [&](int jj, int t) { return t0 + jj * pc.kvs + (pc.kvs == 2 ? t : 0); };
         if (qk_role) {
           // Q K^T(j) of query tile t goes out once S(j-1) of that tile has
           // been read; the Q tiles are released after the piece's last one,
           // each stage after the Q K^T of both tiles has read its K.
           ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, WAIT_NS);
           for (int jj = 0; jj < n && ok; ++jj) {
-            const int tq = t0 + jj, st = tq % STAGES;
-            ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, WAIT_NS);
-            const uint32_t kaddr = smem_addr(sm.k[st]);
             for (int t = 0; t < ntiles && ok; ++t) {
+              const int tq = use_of(jj, t), st = tq % STAGES;
+              if (t == 0 || pc.kvs == 2) {  // the stage holding this tile's K
+                ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, WAIT_NS);
+                if (!ok) break;
+              }
               if (jj > 0) {
                 ok = mbar_wait(smem_addr(&sm.s_free[t]), (t ? ph1 : ph0) & 1, abort_flag, WAIT_NS);
                 if (t) ++ph1; else ++ph0;
@@ -278,13 +292,14 @@ __global__ void __launch_bounds__(THREADS, 1)
               }
               tc_fence_after();
               const uint32_t sq = smem_addr(sm.q[t]), d_s = tmem + (t ? TM_S1 : TM_S0);
+              const uint32_t kaddr = smem_addr(sm.k[st]);
 #pragma unroll
               for (int kk = 0; kk < HD / 16; ++kk)
                 mma_ss(d_s, sdesc_sw128(sq + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
               mma_commit(smem_addr(&sm.s_full[t]));
+              // the stage's K is read by the last Q K^T that uses it
+              if (t == ntiles - 1 || pc.kvs == 2) mma_commit(smem_addr(&sm.kv_empty[st]));
             }
-            if (!ok) break;
-            mma_commit(smem_addr(&sm.kv_empty[st]));
           }
           mma_commit(smem_addr(&sm.q_empty));
           // the softmax also arrives on s_free for the piece's last tile; the
@@ -295,14 +310,14 @@ __global__ void __launch_bounds__(THREADS, 1)
             ok = mbar_wait(smem_addr(&sm.s_free[1]), ph1 & 1, abort_flag, WAIT_NS);
             ++ph1;
           }
-        } else if (tpv == 0 || pc.has1) {
+        } else if (tpv == 0 || pc.ut.has1) {
           // P V(j) of the query tile goes out once P(j) is stored; the stage
           // is released when it completes (the last read of its V)
           const uint32_t b_pready = smem_addr(&sm.p_ready[tpv]), b_odone = smem_addr(&sm.o_done[tpv]);
           const uint32_t f_pub = smem_addr(&sm.flag_o[tpv]);
           const uint32_t d_o = tmem + (tpv ? TM_O1 : TM_O0), d_p = tmem + (tpv ? TM_P1 : TM_P0);
           for (int jj = 0; jj < n && ok; ++jj) {
-            const int st = (t0 + jj) % STAGES;
+            const int st = use_of(jj, tpv) % STAGES;
             ok = mbar_wait(b_pready, ph0 & 1, abort_flag, WAIT_NS);
             ++ph0;
             if (!ok) {
@@ -323,13 +338,20 @@ __global__ void __launch_bounds__(THREADS, 1)
             ++ph1;
             ok = done;
             st_release_shared(f_pub, done ? ph1 : FLAG_ABORT);
+            if (ok && pc.kvs == 2) {
+              // the other head's stage of this key tile: this issuer's release
+              // of it (an arrival only after that use's load has landed)
+              const int to = use_of(jj, 1 - tpv), so = to % STAGES;
+              ok = mbar_wait(smem_addr(&sm.kv_full[so]), (to / STAGES) & 1, abort_flag, WAIT_NS);
+              if (ok) mbar_arrive(smem_addr(&sm.kv_empty[so]));
+            }
           }
         } else {
           // tile 1 of a unit without one: nothing to compute, but the stage
           // releases keep their order (an arrival for a stage's next use
           // only after that use's load has landed)
           for (int jj = 0; jj < n && ok; ++jj) {
-            const int tq = t0 + jj, st = tq % STAGES;
+            const int tq = use_of(jj, 0), st = tq % STAGES;
             ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, WAIT_NS);
             if (ok) mbar_arrive(smem_addr(&sm.kv_empty[st]));
           }
@@ -389,7 +411,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       const Piece pc = piece_at(p, x, x_end);
       const int n = pc.j1 - pc.j0;
       x += n;
-      if (t == 1 && !pc.has1) continue;  // no rows in this unit's second tile
+      if (t == 1 && !pc.ut.has1) continue;  // no rows in this unit's second tile
+      const int th = t ? pc.ut.h1 : pc.ut.h0, tqt = t ? pc.ut.qt1 : pc.ut.qt0;  // this tile's head, index
       float m_used = -INFINITY;  // running max of the logits, scaled to log2 units
       float l = 0.f;             // running row sum of exp2(z*c - m_used)
       for (int jj = 0; jj < n; ++jj) {
@@ -489,10 +512,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       tc_fence_before();
       const float inv_l = 1.f / l;
       const float lse_val = (m_used + __log2f(l)) * 0.69314718055994531f;
-      const int q = (2 * pc.qp + t) * BM + row;
+      const int q = tqt * BM + row;
       if (pc.j0 == 0 && pc.j1 == p.nkv) {
         if (q < p.N) {
-          uint4* dst = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + pc.h) * HD);
+          uint4* dst = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + th) * HD);
 #pragma unroll
           for (int c8 = 0; c8 < 8; ++c8) {
             uint4 w;
@@ -502,7 +525,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             w.w = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 6]) * inv_l, __uint_as_float(orr[c8 * 8 + 7]) * inv_l);
             dst[c8] = w;
           }
-          p.lse[(size_t)pc.h * p.N + q] = lse_val;
+          p.lse[(size_t)th * p.N + q] = lse_val;
         }
       } else {
         // a piece of a unit split between CTAs: its normalised partial goes
@@ -563,8 +586,7 @@ Params make_params(const AttnArgs& a) {
   const int nf = (a.N + BN - 1) / BN;
   p.nkv = p.nb + nf;
   p.nqt = (a.N + BM - 1) / BM;
-  p.nqp = (p.nqt + 1) / 2;
-  p.total = (long long)a.H * p.nqp * p.nkv;
+  p.total = attn_units(p.nqt, a.H) * p.nkv;
   p.scale_log2 = a.scale * 1.4426950408889634f;
   p.out = a.out;
   p.lse = a.lse;
@@ -584,7 +606,6 @@ SplitLayout attn_split_layout(const AttnArgs& a) {
   l.total = p.total;
   l.G = a.grid;
   l.nkv = p.nkv;
-  l.nqp = p.nqp;
   l.nqt = p.nqt;
   l.N = a.N;
   l.H = a.H;
@@ -597,7 +618,7 @@ SplitLayout attn_split_layout(const AttnArgs& a) {
 
 AttnPlan attn_plan(int N, int H, int M) {
   AttnPlan pl;
-  pl.units = (long long)H * (((N + BM - 1) / BM + 1) / 2);
+  pl.units = attn_units((N + BM - 1) / BM, H);
   pl.tiles_per_unit = (M + BN - 1) / BN + (N + BN - 1) / BN;
   pl.total = pl.units * pl.tiles_per_unit;
   return pl;

@@ -43,7 +43,7 @@ struct SplitLayout {
   long long total;        // units * nkv
   int G;                  // attention CTAs
   int nkv;                // key tiles per unit
-  int nqp, nqt;           // query-tile pairs (units) per head, query tiles per head
+  int nqt;                // query tiles per head
   int N, H;
   const __nv_bfloat16* part_o;  // [G][2][kUnitRows][64] piece partials (bf16)
   const float* part_lse;  // [G][2][kUnitRows]
@@ -72,9 +72,47 @@ struct AttnArgs {
   unsigned long long* clk_end;
 };
 
-// Work decomposition: a unit is (head, pair of 128-row query tiles); each
-// unit runs over all key tiles of [bank ; frame].
+// Work decomposition: a unit is a pair of 128-row query tiles run over all
+// key tiles of [bank ; frame]: two consecutive tiles of one head, or, when a
+// head has an odd number of query tiles, the last (lone) tiles of heads 2g
+// and 2g + 1 together (a lone tile's softmax warpgroup paces its chain alone
+// and leaves the tensor core idle half the time; paired, the two tiles keep
+// it busy as a same-head pair does, at the cost of loading both heads' K/V).
+// With an odd head count the last head's lone tile stays a unit by itself.
+// Units are ordered by pairs of heads: head 2g's pairs, head 2g + 1's pairs,
+// then their lone tiles, so units that read the same K/V run close in time.
 constexpr int kUnitRows = 2 * kTile;
+struct UnitTiles {
+  int h0, qt0;  // head and query tile of the unit's first tile
+  int h1, qt1;  // of its second tile (qt1 = qt0 + 1 past the last tile when has1 is false)
+  bool has1;    // the second tile holds rows
+};
+__host__ __device__ inline long long attn_units(int nqt, int H) {
+  return (long long)H * (nqt >> 1) + ((nqt & 1) ? (H + 1) / 2 : 0);
+}
+__host__ __device__ inline UnitTiles unit_tiles(long long u, int nqt, int H) {
+  const int nfp = nqt >> 1, odd = nqt & 1;
+  const int gs = 2 * nfp + odd;  // units of a group of two heads
+  const int g = (int)(u / gs), r = (int)(u - (long long)g * gs);
+  const bool two = 2 * g + 1 < H;  // the group has two heads (else: the last head alone)
+  UnitTiles ut;
+  ut.has1 = true;
+  if (r < nfp || (two && r < 2 * nfp)) {  // a same-head pair
+    ut.h0 = ut.h1 = 2 * g + (r >= nfp ? 1 : 0);
+    ut.qt0 = 2 * (r >= nfp ? r - nfp : r);
+    ut.qt1 = ut.qt0 + 1;
+  } else if (two) {  // the lone tiles of heads 2g and 2g + 1
+    ut.h0 = 2 * g;
+    ut.h1 = 2 * g + 1;
+    ut.qt0 = ut.qt1 = nqt - 1;
+  } else {  // the last head's lone tile (odd head count)
+    ut.h0 = ut.h1 = 2 * g;
+    ut.qt0 = nqt - 1;
+    ut.qt1 = nqt;
+    ut.has1 = false;
+  }
+  return ut;
+}
 struct AttnPlan {
   long long units, tiles_per_unit, total;
 };

@@ -1,7 +1,7 @@
 // The attention's stream-K split and the merge of units cut between CTAs.
 //
-// The (unit, key tile) sequence -- a unit is (head, pair of 128-row query
-// tiles), run over every key tile of [bank ; frame] -- is cut into G
+// The (unit, key tile) sequence -- a unit is a pair of 128-row query tiles
+// (unit_tiles), run over every key tile of [bank ; frame] -- is cut into G
 // contiguous equal ranges, CTA b taking [b T / G, (b + 1) T / G).  A unit cut
 // by a CTA boundary leaves, from each CTA that holds part of it, one
 // normalised partial per query row, (O_p, LSE_p), in the CTA's slot 0 (the
@@ -62,8 +62,9 @@ __device__ __forceinline__ size_t piece_row(const Pieces& pc, int i, int r) {
 // units before the fp32 fold.
 __device__ __forceinline__ void merge_row(const Layout& s, const Pieces& pc, int u, int t, int r,
                                           int qtr) {
-  const int h = u / s.nqp, qp = u - h * s.nqp;
-  const int q = (2 * qp + t) * kRows + r;
+  const UnitTiles ut = unit_tiles(u, s.nqt, s.H);
+  const int h = t ? ut.h1 : ut.h0;
+  const int q = (t ? ut.qt1 : ut.qt0) * kRows + r;
   const int ur = t * kRows + r;  // row within the unit
   const int np = pc.b_hi - pc.b_lo + 1;
   // the partials were kept in L2 for this read; afterwards they may go
@@ -146,8 +147,7 @@ __device__ __forceinline__ Job prepare_job(const Layout& s, int j) {
   const int u = (int)(xb / s.nkv);
   const long long x0 = (long long)u * s.nkv;
   if (xb == x0 || range_begin(bnd - 1, s.G, s.total) > x0) return jb;
-  const int qp = u % s.nqp;
-  if (jb.t == 1 && 2 * qp + 1 >= s.nqt) return jb;
+  if (jb.t == 1 && !unit_tiles(u, s.nqt, s.H).has1) return jb;
   jb.u = u;
   jb.pc.b_lo = bnd - 1;  // the CTA holding the unit's first tile
   jb.pc.b_hi = cta_of(x0 + s.nkv - 1, s.G, s.total);

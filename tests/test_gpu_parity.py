@@ -126,7 +126,10 @@ def test_teacher_forced_bank_lengths(M):
     (1, 1, 8, 8, 20352),   # 160 key tiles on the grid: one or two tiles per CTA
     (1, 1, 8, 8, 40000),   # one unit split over every CTA of the grid
     (2, 4, 14, 14, 30000),  # two query tiles per unit, each unit over half the grid
-    (3, 5, 37, 37, 5000),  # eleven query tiles: the last unit of each head has one
+    (3, 5, 37, 37, 5000),  # eleven query tiles: heads 0 and 1 share a unit of their last
+                           # tiles, head 2's last tile is a unit by itself
+    (2, 1, 8, 8, 30000),   # one query tile per head: a single two-head unit over the grid
+    (4, 5, 37, 37, 12000),  # two two-head units, each split over many CTAs
 ])
 def test_split_units_across_many_ctas(H, ns, gh, gw, M):
     """Few heads and a long bank: units whose key tiles are spread over many
