@@ -65,9 +65,9 @@ CONFIGS = {
 # (frame 1001 of the 2000-frame stream, L = 16,734: 71.75 MB read + 1.95 MB
 # written).  Set back to None whenever the
 # attention kernel changes until it is captured again.
-ATTN_TRAFFIC_BYTES_PER_LAUNCH = 74.99e6
+ATTN_TRAFFIC_BYTES_PER_LAUNCH = 76.25e6
 ATTN_TRAFFIC_NOTE = ("ncu dram bytes of the frame-1001 launch (mean attended length of the "
-                     "stream); the frame-2000 launch moves 562.6 MB (L2 no longer holds a "
+                     "stream); the frame-2000 launch moves 497.0 MB (L2 no longer holds a "
                      "layer's bank)")
 
 
