@@ -154,6 +154,41 @@ def test_split_units_across_many_ctas(H, ns, gh, gw, M):
         st.close()
 
 
+def test_running_max_renewed_by_large_later_logits():
+    """A row's running max grows by far more than the softmax lets it lag
+    (2^8 in exp2 units) after its piece's first key tiles: a bank whose first
+    600 rows are tiny and whose rows 1500-1503 are 50 * ones gives logits up
+    to ~10^3 above the first tiles' maximum in the rows where sum(q) is
+    large, so those rows rescale O and l mid-piece (in pieces that start
+    before the large rows; pieces starting after them take the large max on
+    their first tile).  All rows must still match the oracle."""
+    H, ns, gh, gw, M = 2, 5, 37, 37, 2000
+    st = Stream(1, H, ns, gh, gw, budget=14, max_frames=M // 14 + 2, seed=9)
+    try:
+        g = torch.Generator().manual_seed(99)
+        bk = torch.randn(H, M, 64, generator=g)
+        bk[:, :600] *= 0.05
+        bk[:, 1500:1502] = 50.0
+        bk[:, 1502:1504, ::2] = 50.0  # a second large row in the other half of its tile
+        bk = bk.to(torch.bfloat16)
+        bv = torch.randn(H, M, 64, generator=g).to(torch.bfloat16)
+        st.rm.import_bank(0, bk, bv, M)
+        q, k, v = st.inputs(0, 3)
+        out, sal, lse = st.attend(0, q, k, v)
+        torch.cuda.synchronize()
+        ref = orc.attend_frame(to64(q), to64(k), to64(v), [bk[h].double().numpy() for h in range(H)],
+                               [bv[h].double().numpy() for h in range(H)], 1 / 8,
+                               orc.sampled_query_tokens(ns, gh, gw, 2))
+        # the case is only meaningful if many rows' logits outgrow the first tiles' by far
+        z_big = to64(q)[:, 0, :].sum(axis=1) * 50.0 / 8.0
+        assert (z_big * 1.4426950408889634 > 64 + 5).sum() > 50
+        check_o(out, ref["O"], "renewed running max")
+        check_lse(lse, ref["LSE"], "renewed running max")
+        check_saliency(sal, ref["S"], "renewed running max")
+    finally:
+        st.close()
+
+
 def test_long_bank_sampled_rows():
     """Config-4 end size: a bank of 29360 rows per head (2000 frames at k = 14).
     O is checked on sampled query rows (the oracle computes rows one by one),
