@@ -175,7 +175,9 @@ REGMEM_API regmem_status regmem_admit_shared(regmem_t* h, int32_t layer, int32_t
  * and errors as in the two
  * calls; every check (including k and capacity) is made before anything is
  * enqueued.  The library keeps no pointer after the call: K, V and saliency
- * need only stay valid until the enqueued work has run.
+ * need only stay valid until the enqueued work has run (with overlap, that
+ * includes the side stream's saliency and admission: regmem_synchronize or
+ * regmem_join).
  * State: the layer must not have an attend pending (ERR_STATE); afterwards
  * it has none. */
 REGMEM_API regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, const void* K,
@@ -189,8 +191,8 @@ REGMEM_API regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const v
  * call's host->device copies overlap the previous call's kernels and its
  * device->host copies the next call's.  Host buffers should be pinned (pageable ones are copied
  * synchronously by CUDA).  The caller must not modify hostQ/hostK/hostV, nor
- * read hostOut/hostSaliency, before regmem_synchronize (which waits for both
- * streams); consecutive calls may reuse the same buffers. */
+ * read hostOut/hostSaliency, before regmem_synchronize (which waits for all
+ * of the handle's streams); consecutive calls may reuse the same buffers. */
 REGMEM_API regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* hostQ,
                                        const void* hostK, const void* hostV, void* hostOut,
                                        float* hostSaliency, int32_t k);
