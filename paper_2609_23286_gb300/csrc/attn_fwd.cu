@@ -565,13 +565,20 @@ __global__ void __launch_bounds__(THREADS, 1)
   grid_dep_launch();
 }
 
-// Merges the pieces of every split unit (split.cuh): block j takes merge
-// job j, tile j & 1 of the unit cut by the boundary between CTAs j / 2 and
-// j / 2 + 1.  2 (G - 1) blocks, two per SM: every block is resident at once.
+// Merges the pieces of every split unit (split.cuh): block b takes merge job
+// jobs.j[b], tile j & 1 of the unit cut by the boundary between CTAs j / 2
+// and j / 2 + 1.  Only the jobs that merge something are launched (the host
+// lists them), at most 2 (G - 1) blocks, two per SM: every block is resident
+// at once, and the SMs without a merge block are free for the next kernel.
 constexpr int CMB_THREADS = 4 * BM;
+struct CombineJobs {
+  unsigned short j[2 * kAttnMaxGrid];
+};
 
-__global__ void __launch_bounds__(CMB_THREADS, 2) attn_combine_kernel(const SplitLayout lay) {
-  const split::Job jb = split::prepare_job(lay, blockIdx.x);  // layout only: before the wait
+__global__ void __launch_bounds__(CMB_THREADS, 2)
+    attn_combine_kernel(const SplitLayout lay, const CombineJobs jobs) {
+  const unsigned j = jobs.j[blockIdx.x];
+  const split::Job jb = split::prepare_job(lay, j == 0xFFFFu ? -1 : (int)j);  // layout only: before the wait
   grid_dep_wait();  // every piece's partial is stored
   grid_dep_launch();
   split::run_job<CMB_THREADS>(lay, jb, threadIdx.x);
@@ -652,8 +659,13 @@ cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_b
   if (e != cudaSuccess) return e;
   if (ev_after && (e = cudaEventRecord(ev_after, s)) != cudaSuccess) return e;
   if (a.grid > 1) {  // with one CTA no unit is split
-    e = launch_pdl(attn_combine_kernel, dim3((unsigned)(2 * (a.grid - 1))), dim3(CMB_THREADS), 0, s,
-                   attn_split_layout(a));
+    const SplitLayout lay = attn_split_layout(a);
+    CombineJobs jobs;
+    unsigned n = 0;
+    for (int j = 0; j < 2 * (a.grid - 1); ++j)
+      if (split::job_live(lay, j)) jobs.j[n++] = (unsigned short)j;
+    if (n == 0) jobs.j[n++] = 0xFFFF;  // one block that merges nothing: the launch is counted
+    e = launch_pdl(attn_combine_kernel, dim3(n), dim3(CMB_THREADS), 0, s, lay, jobs);
     if (e != cudaSuccess) return e;
   }
   if (ev_merged && (e = cudaEventRecord(ev_merged, s)) != cudaSuccess) return e;

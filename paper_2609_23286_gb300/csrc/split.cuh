@@ -138,16 +138,23 @@ struct Job {
   int u, t;  // u < 0: nothing to merge
   Pieces pc;
 };
-__device__ __forceinline__ Job prepare_job(const Layout& s, int j) {
-  Job jb;
-  jb.u = -1;
+// Whether job j merges anything (host and device).
+__host__ __device__ inline bool job_live(const Layout& s, int j) {
   const int bnd = j / 2 + 1;
-  jb.t = j & 1;
   const long long xb = range_begin(bnd, s.G, s.total);
   const int u = (int)(xb / s.nkv);
   const long long x0 = (long long)u * s.nkv;
-  if (xb == x0 || range_begin(bnd - 1, s.G, s.total) > x0) return jb;
-  if (jb.t == 1 && !unit_tiles(u, s.nqt, s.H).has1) return jb;
+  if (xb == x0 || range_begin(bnd - 1, s.G, s.total) > x0) return false;
+  return (j & 1) == 0 || unit_tiles(u, s.nqt, s.H).has1;
+}
+__device__ __forceinline__ Job prepare_job(const Layout& s, int j) {
+  Job jb;
+  jb.u = -1;
+  jb.t = j & 1;
+  if (j < 0 || !job_live(s, j)) return jb;
+  const int bnd = j / 2 + 1;
+  const long long x0 = range_begin(bnd, s.G, s.total) / s.nkv * s.nkv;
+  const int u = (int)(x0 / s.nkv);
   jb.u = u;
   jb.pc.b_lo = bnd - 1;  // the CTA holding the unit's first tile
   jb.pc.b_hi = cta_of(x0 + s.nkv - 1, s.G, s.total);
