@@ -185,7 +185,7 @@ REGMEM_API regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const v
                                   int32_t* idx_out);
 
 /* regmem_attend_admit with HOST buffers (layouts as in
- * regmem_attend_frame_host; no index output).  Three library-owned staging
+ * regmem_attend_frame_host; no index output).  Six library-owned staging
  * sets are used in turn and the copies run on two copy streams of the
  * handle's own (one each way), ordered against the kernels by events: a
  * call's host->device copies overlap the previous call's kernels and its

@@ -60,12 +60,14 @@ struct regmem {
   __nv_bfloat16* stOut = nullptr;
   float* stSal = nullptr;
   std::vector<__nv_bfloat16*> stK, stV;
-  // regmem_attend_admit_host: three staging sets used in turn, copies in
-  // and out on streams of their own, so one call's copies overlap the
-  // neighbouring calls' kernels.  Three, not two: with overlap a set's
-  // inputs are read until the call's side work ends, in the next call's
-  // attention, so the inputs of the call after next go to a third set.
-  static constexpr unsigned kHostSets = 3;
+  // regmem_attend_admit_host: six staging sets used in turn, copies in and
+  // out on streams of their own, so one call's copies overlap the
+  // neighbouring calls' kernels.  A set's inputs are read until the call's
+  // side work ends (with overlap, inside the next call's attention) and its
+  // outputs are copied out after that, so a set is free again only a few
+  // calls later: with two sets the input copies waited for it, and six ran
+  // the host-buffer stream faster than three.
+  static constexpr unsigned kHostSets = 6;
   struct HostSet {
     __nv_bfloat16 *q = nullptr, *k = nullptr, *v = nullptr, *out = nullptr;
     float* sal = nullptr;
