@@ -9,8 +9,14 @@ the saliency kernel).
 Default workload: the long-horizon stream -- 24 layers, 16 heads x 64,
 1374 tokens per frame (37x37 patches + 5 special tokens), k = 14 admitted
 rows per head per frame, 2000 frames, so each layer's memory grows from 0 to
-29,360 rows.  `value` is frames/s over the timed frames (frames 1..K of a
-fresh stream, after W warm-up frames on the same handle followed by a reset).
+29,360 rows.  `value` is frames/s over the timed frames.  With --steps K
+shorter than the stream, the K timed frames are a window centred on the
+stream's middle frame, where a frame attends the stream's mean number of
+keys (Eq. 6: the memory grows linearly, so the middle frame's length is the
+mean): frames 991-1010 for K = 20 on the 2000-frame stream.  Each layer's
+bank then starts with the rows that frame would see (seeded synthetic rows
+imported through regmem_import_bank), restored after the W warm-up frames.
+--start-frame overrides the window; --steps 0 times the whole stream.
 
 Inputs: Q/K/V come from a pool of distinct seeded synthetic frames resident
 in HBM (frame t uses pool entry (t-1) mod P); every step touches more than
@@ -18,17 +24,20 @@ L2 holds (>= 202 MB of inputs per frame, plus the banks), so no L2 flush is
 needed.
 
 Also reported:
-  roofline      attention kernel: algorithmic FLOPs / CUDA-event time of its
-                launches in the timed region, against the measured bf16 peak
+  roofline      attention kernel: algorithmic FLOPs / the kernel's own launch
+                clock over every launch of the timed region, against the
+                measured bf16 peak (burst for a timed region under a second,
+                sustained for longer ones)
   e2e           same metric through regmem_attend_admit_host: pinned host
                 Q/K/V in, O and saliency back to host, copies inside the timed
                 region
   cpu_baseline  the fp64 oracle on the host cores, timed on a bounded sample
-                (single layer-frames), extrapolated to the stream
+                of the same frames (single layer-frames at the window's ends,
+                cost linear in the attended length)
   clocks        nvidia-smi samples taken during the timed region
 
---impl reference runs only the oracle (the reference arm) on the same
-workload definition.
+--impl reference runs only the oracle (the reference arm) on the same frames:
+each step is one (layer, head) of a layer-frame of the window.
 Under torchrun with --gpus N each rank runs an independent replica stream
 (distinct seed): weak scaling, no collective on the data path.
 """
@@ -61,14 +70,57 @@ CONFIGS = {
 }
 
 # dram__bytes_read.sum + dram__bytes_write.sum of one attention-kernel launch,
-# from an ncu capture of the launch at the stream's mean attended length
-# (frame 1001 of the 2000-frame stream, L = 16,734: 71.75 MB read + 1.95 MB
-# written).  Set back to None whenever the
-# attention kernel changes until it is captured again.
-ATTN_TRAFFIC_BYTES_PER_LAUNCH = 76.25e6
-ATTN_TRAFFIC_NOTE = ("ncu dram bytes of the frame-1001 launch (mean attended length of the "
-                     "stream); the frame-2000 launch moves 497.0 MB (L2 no longer holds a "
-                     "layer's bank)")
+# from ncu captures of single launches (profiles/attn_fwd_long_stream.md):
+# {(config, attended rows L): bytes}.  The line reports the capture whose L
+# lies within 2 % of the timed launches' mean L, else null; the table is
+# emptied whenever the attention kernel changes until it is captured again.
+ATTN_TRAFFIC_CAPTURES = {}
+
+
+def traffic_for(cfg_name, mean_L):
+    """(bytes per launch, note) of a capture matching the timed launches."""
+    for (name, L), b in ATTN_TRAFFIC_CAPTURES.items():
+        if name == cfg_name and abs(L - mean_L) <= 0.02 * mean_L:
+            return b, (f"ncu dram bytes (read + write) of one attention launch at L = {L} "
+                       f"(timed launches: mean L = {mean_L:.0f})")
+    return None, "no ncu capture of the attention kernel at this attended length"
+
+
+def default_start_frame(frames, K):
+    """First timed frame: K frames centred on the stream's middle frame, whose
+    attended length is the stream's mean (the memory grows linearly, Eq. 6);
+    the whole stream when K covers it."""
+    if K <= 0 or K >= frames:
+        return 1
+    mid = frames // 2 + 1
+    return max(1, min(mid - K // 2, frames - K + 1))
+
+
+def window_frames(S0, K):
+    return list(range(S0, S0 + K))
+
+
+def mean_attended(cfg, frames):
+    Ls = [attended_rows(cfg, t, l) for t in frames for l in range(cfg["layers"])]
+    return sum(Ls) / len(Ls)
+
+
+def bench_config(cfg, name, S0, K, world):
+    """The `config` object, identical in both arms' lines."""
+    frames = window_frames(S0, K)
+    return {
+        "workload": describe(cfg, name),
+        "first_frame": S0,
+        "frames_timed": K,
+        "stream_frames": cfg["frames"],
+        "mean_attended_rows": round(mean_attended(cfg, frames), 1),
+        "window": ("whole stream" if S0 == 1 and K >= cfg["frames"] else
+                   f"frames {S0}-{S0 + K - 1} of the stream, banks pre-filled with the rows "
+                   "those frames see"),
+        "l2": "no flush: inputs larger than L2 (>= 202 MB of Q/K/V per step plus the banks)",
+        "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+        **({"variant": cfg["variant"]} if cfg.get("variant") else {}),
+    }
 
 
 # Attention launches bracketed by CUDA events inside the timed region: every
@@ -237,11 +289,14 @@ def oracle_layer_frame_seconds(cfg, t, heads=None, seed=7):
     return time.perf_counter() - t0
 
 
-def oracle_baseline(cfg):
-    """Bounded CPU baseline: single layer-frames at a few stream positions,
-    cost fitted linear in the attended length L and summed over the stream."""
-    frames = cfg["frames"]
-    ts = sorted(set([2, max(2, frames // 2 + 1), frames]))
+def oracle_baseline(cfg, S0, K):
+    """Bounded CPU baseline on the timed frames S0 .. S0+K-1: single
+    layer-frames (all heads) at the window's first and last frame, cost
+    fitted linear in the attended length L and summed over the window's
+    layer-frames (plus, with frame-attention layers, one frame-attention
+    layer-frame timed at L = N for each)."""
+    frames = window_frames(S0, K)
+    ts = sorted(set([frames[0], frames[-1]]))
     pts = [(attended_rows(cfg, t), oracle_layer_frame_seconds(cfg, t)) for t in ts]
     if len(pts) >= 2:
         (l0, s0), (l1, s1) = pts[0], pts[-1]
@@ -249,17 +304,21 @@ def oracle_baseline(cfg):
         b = s0 - a * l0
     else:
         a, b = pts[0][1] / pts[0][0], 0.0
-    total = sum(max(a * attended_rows(cfg, t) + b, 0.0) for t in range(1, frames + 1))
-    total *= cfg["layers"] * (2 if cfg["fa"] else 1)
-    return {"frames_per_s": frames / total, "samples": pts}
+    total = sum(max(a * attended_rows(cfg, t, l) + b, 0.0)
+                for t in frames for l in range(cfg["layers"]))
+    fa = None
+    if cfg["fa"]:
+        fa = oracle_layer_frame_seconds(cfg, 1)
+        total += fa * cfg["layers"] * len(frames)
+    return {"frames_per_s": len(frames) / total, "samples": pts, "frame_attention_s": fa}
 
 
-def run_oracle_subprocess(cfg, what="baseline", steps=0, warmup=0):
+def run_oracle_subprocess(cfg, what="baseline", steps=0, warmup=0, S0=1, K=1):
     threads = os.cpu_count() or 1
     env = dict(os.environ, OPENBLAS_NUM_THREADS=str(threads), OMP_NUM_THREADS=str(threads),
                MKL_NUM_THREADS=str(threads), CUDA_VISIBLE_DEVICES="")
     code = (f"import json, bench; print(json.dumps(bench._oracle_entry({json.dumps(cfg)!r}, "
-            f"{what!r}, {steps}, {warmup})))")
+            f"{what!r}, {steps}, {warmup}, {S0}, {K})))")
     r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True,
                        text=True)
     if r.returncode != 0:
@@ -269,17 +328,27 @@ def run_oracle_subprocess(cfg, what="baseline", steps=0, warmup=0):
     return out
 
 
-def _oracle_entry(cfg_json, what, steps, warmup):
+def _oracle_entry(cfg_json, what, steps, warmup, S0, K):
     cfg = json.loads(cfg_json)
     if what == "baseline":
-        return oracle_baseline(cfg)
-    # reference arm: each step = one (layer, head) of a layer-frame at the
-    # stream's middle frame (mean attended length)
-    t_mid = cfg["frames"] // 2 + 1
-    for _ in range(warmup):
-        oracle_layer_frame_seconds(cfg, t_mid, heads=1)
-    times = [oracle_layer_frame_seconds(cfg, t_mid, heads=1, seed=11 + i) for i in range(steps)]
-    return {"step_s": times, "t_mid": t_mid}
+        return oracle_baseline(cfg, S0, K)
+    # reference arm: step i = one (layer, head) of a layer-frame at frame
+    # S0 + (i mod K) of the timed window (plus, with frame-attention layers,
+    # one (layer, head) of a frame-attention layer-frame)
+    frames = window_frames(S0, K)
+    # with fewer steps than timed frames, the steps spread evenly over them
+    picks = [frames[(i * len(frames)) // max(steps, 1)] for i in range(steps)]
+
+    def step(t, seed):
+        s = oracle_layer_frame_seconds(cfg, t, heads=1, seed=seed)
+        if cfg["fa"]:
+            s += oracle_layer_frame_seconds(cfg, 1, heads=1, seed=seed + 1)
+        return s
+
+    for i in range(warmup):
+        step(picks[i % len(picks)] if picks else frames[0], 5)
+    times = [step(t, 11 + i) for i, t in enumerate(picks)]
+    return {"step_s": times, "frames": picks}
 
 
 # ---------------------------------------------------------------------------
@@ -333,6 +402,18 @@ def synthetic_bank(cfg, rows, seed, device):
     return k.to(torch.bfloat16).cpu(), v.to(torch.bfloat16).cpu()
 
 
+def timed_window(args, cfg):
+    """(first timed frame, frames timed) for the command line: --start-frame
+    if given, else the window centred on the stream's middle frame."""
+    if args.steps:
+        K = args.steps
+        S0 = args.start_frame if args.start_frame else default_start_frame(cfg["frames"], K)
+    else:
+        S0 = args.start_frame or 1
+        K = max(cfg["frames"] - S0 + 1, 1)
+    return S0, K
+
+
 def gpu_arm(args, cfg, cfg_name):
     import torch
     import torch.distributed as dist
@@ -350,15 +431,14 @@ def gpu_arm(args, cfg, cfg_name):
               else torch.cuda.current_stream())
     N = cfg["ns"] + cfg["gh"] * cfg["gw"]
     H, L = cfg["heads"], cfg["layers"]
-    S0 = args.start_frame
-    K = args.steps if args.steps else cfg["frames"] - S0 + 1
+    S0, K = timed_window(args, cfg)
     W = args.warmup
     seed = cfg["seed"] + 1000 * rank
 
     # CPU baseline first (fresh process, before this process's GPU work grows)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        cpu = run_oracle_subprocess(cfg, "baseline")
+        cpu = run_oracle_subprocess(cfg, "baseline", S0=S0, K=K)
 
     P = min(args.pool, max(K, W, 1))
     pool = make_pool(cfg, P, seed, dev)
@@ -422,21 +502,29 @@ def gpu_arm(args, cfg, cfg_name):
         hout = torch.empty(N, H, 64, dtype=torch.bfloat16).pin_memory()
         hsal = torch.empty(H, N, dtype=torch.float32).pin_memory()
         hfa = torch.empty_like(hout).pin_memory() if cfg["fa"] else None
+
+        def host_frames(t0, count):
+            for t in range(t0, t0 + count):
+                for layer in range(L):
+                    q, k, v = hpool[layer][(t - 1) % Ph]
+                    if hfa is not None:
+                        fq, fk, fv = pool[layer][t % P]
+                        rm.frame_attention(fq, fk, fv, fa_out)  # frame-attention layer: device inputs
+                    rm.attend_admit_host(layer, q, k, v, hout, hsal, layer_k(cfg, layer))
+
+        # untimed warm-up frames through the host path, then the same banks
+        # as the device leg's timed region
         restore()
         rm.profile_enable(0)
+        host_frames(S0, W)
         rm.synchronize()
+        restore()
         barrier()
         torch.cuda.synchronize()
         # host clock around the calls and the final synchronisation: the
         # library's copies run on a stream of its own
         t_e0 = time.perf_counter()
-        for t in range(S0, S0 + K):
-            for layer in range(L):
-                q, k, v = hpool[layer][(t - 1) % Ph]
-                if hfa is not None:
-                    fq, fk, fv = pool[layer][t % P]
-                    rm.frame_attention(fq, fk, fv, fa_out)  # frame-attention layer: device inputs
-                rm.attend_admit_host(layer, q, k, v, hout, hsal, layer_k(cfg, layer))
+        host_frames(S0, K)
         t_enq = time.perf_counter()
         rm.synchronize()
         e2e_ms = max_over_ranks((time.perf_counter() - t_e0) * 1e3, dev)
@@ -461,9 +549,16 @@ def gpu_arm(args, cfg, cfg_name):
         pass
     peak_sust = peaks.get("bf16_tflops_sustained")
     peak_burst = peaks.get("bf16_tflops")
-    peak_src = "measured (MEASURED_PEAKS.json bf16_tflops_sustained: kernel timed inside a long step)"
-    if peak_sust is None:
-        peak_sust, peak_burst, peak_src = 1700.0, 1900.0, "fallback"
+    measured = peak_sust is not None and peak_burst is not None
+    if not measured:
+        peak_sust, peak_burst = 1700.0, 1900.0
+    # the burst peak for a timed region shorter than a second (the GPU has no
+    # time to settle under its power cap), the sustained one for longer runs
+    long_run = ms >= 1000.0
+    peak = peak_sust if long_run else peak_burst
+    peak_src = ("measured" if measured else "fallback") + (
+        " bf16 sustained peak (timed region >= 1 s)" if long_run
+        else " bf16 burst peak (timed region < 1 s)")
     attn_tflops = prof.attention_flops / (prof.attention_ms / 1e3) / 1e12 if prof.attention_ms else 0.0
     attn_ms_mean = prof.attention_ms / max(prof.attention_timed, 1)
     if prof.attention_clocked:
@@ -479,6 +574,7 @@ def gpu_arm(args, cfg, cfg_name):
     if cfg["fa"]:
         flops_total += 4.0 * N * N * 64 * H * L * K
     clk = clocks.summary()
+    traffic = traffic_for(cfg_name, mean_attended(cfg, window_frames(S0, K)))
     line = {
         "metric": METRIC,
         "value": round(K * world / (ms / 1e3), 3),
@@ -492,17 +588,13 @@ def gpu_arm(args, cfg, cfg_name):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) Q/K/V, log-normal(0,0.5) per-token key scale, bf16)",
-        "config": {
-            "workload": describe(cfg, cfg_name),
-            "frames_timed": K,
-            "first_frame": S0,
-            "stream_frames": cfg["frames"],
+        "config": bench_config(cfg, cfg_name, S0, K, world),
+        "run": {
             "final_memory_rows_per_head": mem_rows,
             "input_pool_frames": P,
-            "l2": "no flush: inputs larger than L2 (>= 202 MB of Q/K/V per step plus the banks)",
-            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
             "overlap": ("saliency + admission on a side stream" if args.overlap
                         else "all kernels on one stream"),
+            "timed_region_ms": round(ms, 3),
         },
         "tflops_attention_path": round(flops_total / (ms / 1e3) / 1e12 * world, 2),
         "roofline": {
@@ -513,15 +605,16 @@ def gpu_arm(args, cfg, cfg_name):
             # CTA's end): nothing is recorded between launches, so no launch
             # loses its programmatic overlap with the previous kernel
             "achieved": round(roof_tflops, 2),
-            "peak": peak_sust,
+            "peak": peak,
             "unit": "TFLOP/s",
-            "frac": round(roof_tflops / peak_sust, 4) if peak_sust else None,
-            "frac_of_burst_peak": round(roof_tflops / peak_burst, 4) if peak_burst else None,
+            "frac": round(roof_tflops / peak, 4),
+            "frac_of_burst_peak": round(roof_tflops / peak_burst, 4),
+            "frac_of_sustained_peak": round(roof_tflops / peak_sust, 4),
             "peak_source": peak_src,
             "timing": ("launch clock: every attention launch, device global timer"
                        if prof.attention_clocked else "CUDA events on sampled launches"),
-            "traffic": ATTN_TRAFFIC_BYTES_PER_LAUNCH,
-            "traffic_note": ATTN_TRAFFIC_NOTE if ATTN_TRAFFIC_BYTES_PER_LAUNCH else None,
+            "traffic": traffic[0],
+            "traffic_note": traffic[1],
             "launches": prof.attention_clocked or prof.attention_timed,
             "launches_total": prof.launches_attention,
             "ctas": prof.attention_ctas,
@@ -536,7 +629,7 @@ def gpu_arm(args, cfg, cfg_name):
             # so these sampled launches run longer than the unobserved ones
             "events": {
                 "achieved": round(attn_tflops, 2),
-                "frac": round(attn_tflops / peak_sust, 4) if peak_sust else None,
+                "frac": round(attn_tflops / peak, 4),
                 "launches": prof.attention_timed,
                 "launches_sampled_every": every,
                 "mean_launch_ms": round(attn_ms_mean, 5),
@@ -552,7 +645,6 @@ def gpu_arm(args, cfg, cfg_name):
     }
     if cfg.get("variant"):
         share = line["roofline"]["share_of_step"] or 0.0
-        line["config"]["variant"] = cfg["variant"]
         line["memory"] = {
             "bank_rows_per_layer": mem_rows_layers,
             "bank_bytes": int(sum(mem_rows_layers) * H * 64 * 2 * 2),
@@ -563,9 +655,12 @@ def gpu_arm(args, cfg, cfg_name):
         line["cpu_baseline"] = {
             "value": round(cpu["frames_per_s"], 6), "unit": UNIT, "cores": cpu["threads"],
             "kind": "oracle",
-            "sample": ("fp64 numpy oracle on single layer-frames at stream frames "
+            "sample": ("fp64 numpy oracle, one layer-frame (all heads) at each end of the "
+                       "timed window: "
                        + ", ".join(f"L={l} ({s:.2f}s)" for l, s in cpu["samples"])
-                       + f"; cost fitted linear in L and summed over {cfg['frames']} frames x "
+                       + (f", frame attention L={N} ({cpu['frame_attention_s']:.2f}s)"
+                          if cpu.get("frame_attention_s") else "")
+                       + f"; cost fitted linear in L and summed over the {K} timed frames x "
                        f"{L} layers; BLAS matmuls on {cpu['threads']} threads, "
                        "elementwise exp single-threaded"),
         }
@@ -576,23 +671,28 @@ def reference_arm(args, cfg, cfg_name):
     rank, _, world = dist_env()
     if rank != 0:
         return None
-    K = args.steps if args.steps else 5
+    S0, Kw = timed_window(args, cfg)
+    steps = args.steps if args.steps else 5
     W = args.warmup
-    r = run_oracle_subprocess(cfg, "reference", K, W)
+    r = run_oracle_subprocess(cfg, "reference", steps, W, S0=S0, K=Kw)
     step = statistics.mean(r["step_s"])
-    units = cfg["layers"] * cfg["heads"] * (2 if cfg["fa"] else 1)
+    units = cfg["layers"] * cfg["heads"]
     fps = 1.0 / (step * units)
+    fr = r["frames"]
+    what = "one (layer, head) of a regulated layer-frame" + (
+        " plus one (layer, head) of a frame-attention layer-frame" if cfg["fa"] else "")
     return {
         "impl": "reference",
         "metric": METRIC, "value": round(fps, 8), "unit": UNIT, "n_gpus": world,
-        "steps": K, "warmup": W, "ms_per_step": round(step * 1e3, 3),
+        "steps": steps, "warmup": W, "ms_per_step": round(step * 1e3, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic", "config": {"workload": describe(cfg, cfg_name)},
+        "data": "synthetic (seeded N(0,1) Q/K/V, log-normal(0,0.5) per-token key scale, bf16)",
+        "config": bench_config(cfg, cfg_name, S0, Kw, world),
         "cpu_baseline": {"kind": "oracle", "cores": r["threads"], "value": round(fps, 8),
                          "unit": UNIT,
-                         "sample": (f"each step = one (layer, head) of a layer-frame at frame "
-                                    f"{r['t_mid']} (mean attended length "
-                                    f"{attended_rows(cfg, r['t_mid'])}); frames/s = 1 / "
+                         "sample": (f"fp64 numpy oracle; each step = {what} at frames "
+                                    f"{fr[0]}..{fr[-1]} of the timed window (mean attended "
+                                    f"length {mean_attended(cfg, fr):.0f}); frames/s = 1 / "
                                     f"({units} x mean step time)")},
         "e2e": {"value": round(fps, 8), "unit": UNIT, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
@@ -607,8 +707,9 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", choices=sorted(CONFIGS), default="long")
     ap.add_argument("--pool", type=int, default=16, help="distinct input frames kept in HBM")
-    ap.add_argument("--start-frame", type=int, default=1,
-                    help="first timed frame; banks are pre-filled with the rows it would see")
+    ap.add_argument("--start-frame", type=int, default=0,
+                    help="first timed frame (default: a window centred on the stream's middle "
+                         "frame); banks are pre-filled with the rows it would see")
     ap.add_argument("--layers", type=int, default=0, help="override the config's layer count")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -665,8 +766,8 @@ def main(argv=None):
         variant["k_per_layer"] = [layer_k(cfg, l) for l in range(cfg["layers"])]
         cfg["variant"] = variant
         args.no_cpu_baseline = True  # the oracle baseline models the default stream only
-    if args.start_frame < 1:
-        ap.error("--start-frame must be >= 1")
+    if args.start_frame < 0 or args.start_frame > cfg["frames"]:
+        ap.error("--start-frame must be in [1, frames] (0: the default window)")
     if args.impl == "reference":
         line = reference_arm(args, cfg, args.config)
     else:

@@ -82,8 +82,14 @@ REGMEM_API regmem_status regmem_create(regmem_t** out, int32_t layers, int32_t h
                             int32_t budget);
 
 /* Fixes the frame geometry and allocates, on the current CUDA device, the
- * banks ([layers][heads][capacity][64] bf16 for K and for V, zero-filled) and
- * the library's scratch.  Must be called once, before the first attend;
+ * banks ([layers][heads][capacity][64] bf16 for K and for V, zero-filled),
+ * the library's scratch, and the staging buffers, copy streams and events of
+ * the host-buffer entry points (six sets of Q, K, V, out and saliency for
+ * regmem_attend_admit_host; Q, out, saliency and per-layer K and V for
+ * regmem_attend_frame_host: 11.3 MB x 6 + 8.5 MB + 5.6 MB x layers at
+ * N = 1374, 16 heads), so that no later call allocates device memory
+ * (regmem_profile_enable's launch clock excepted, see there).  Must be
+ * called once, before the first attend;
  * ERR_STATE if called again. ERR_UNSUPPORTED if N exceeds 65536 or the
  * number of admission candidates exceeds 8192. */
 REGMEM_API regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd);
@@ -134,7 +140,8 @@ REGMEM_API regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const v
 /* Same as regmem_attend_frame but with HOST buffers: Q, K, V and out are
  * bf16 [N][H][64] and saliency fp32 [H][N] in host memory (pinned for
  * asynchronous copies; pageable also works, synchronously).  K and V are
- * staged into library-owned device buffers that stay valid until admit.
+ * staged into library-owned device buffers (made by regmem_set_frame) that
+ * stay valid until admit.
  * The device->host copies of out and saliency are enqueued on the stream:
  * they are complete after regmem_synchronize (or a sync of the stream). */
 REGMEM_API regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* hostQ,
@@ -250,9 +257,12 @@ REGMEM_API regmem_status regmem_synchronize(regmem_t* h);
  * device bf16 [N][heads][64]; bankK/bankV are the caller's device bank of one
  * layer, bf16 [heads][bank_rows][64], of which the first M rows per head are
  * attended (NULL allowed when M == 0); saliency is device fp32 [heads][N];
- * status is an optional device int32 into which the kernels OR nonzero bits if
- * a bounded device-side wait expires (the caller zeroes it and reads it after
- * synchronising); stream is a cudaStream_t (NULL: legacy default stream).
+ * status is a REQUIRED device (or mapped host) int32 into which the kernels
+ * OR nonzero bits if a bounded device-side wait expires; the caller zeroes it
+ * before the call and reads it after synchronising, and treats out and
+ * saliency as undefined when it is nonzero (there is no handle, so no later
+ * call could report the failure; NULL gives REGMEM_ERR_ARG); stream is a
+ * cudaStream_t (NULL: legacy default stream).
  * All pointers 16-byte aligned (status 4-byte aligned).
  *
  * Scratch: the kernels' split partials, LSE rows and sampled-query list live

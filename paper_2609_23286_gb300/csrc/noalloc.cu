@@ -33,7 +33,6 @@ struct NoAllocScratch {
   float part_lse[(size_t)kMaxCtas * 2 * kUnitRows];
   float lse[kMaxLse];
   int qidx[kMaxSampled];
-  int status;  // device status bits when the caller passes no status word
 };
 
 // 11.9 MB; shared by every call on a device.
@@ -99,7 +98,10 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
                                                      float* saliency, int32_t* status,
                                                      void* stream_) {
   cudaStream_t stream = static_cast<cudaStream_t>(stream_);
-  if (!fd || heads < 1 || !Q || !K || !V || !out || !saliency) return REGMEM_ERR_ARG;
+  // status is required: with no handle there is no later call that could
+  // report an expired device-side wait, so the caller's word is the only
+  // place the kernels can record it
+  if (!fd || heads < 1 || !Q || !K || !V || !out || !saliency || !status) return REGMEM_ERR_ARG;
   const int ds = fd->ds == 0 ? 2 : fd->ds;
   if (fd->n_special < 0 || fd->grid_h < 1 || fd->grid_w < 1 || ds < 1 ||
       fd->n_tokens != fd->n_special + fd->grid_h * fd->grid_w || fd->scale < 0.f ||
@@ -109,7 +111,7 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
     return REGMEM_ERR_ARG;
   if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(out) || !aligned16(saliency) ||
       (M > 0 && (!aligned16(bankK) || !aligned16(bankV))) ||
-      (status && (reinterpret_cast<uintptr_t>(status) & 3u)))
+      (reinterpret_cast<uintptr_t>(status) & 3u))
     return REGMEM_ERR_ARG;
   const int N = fd->n_tokens;
   const int cols = (fd->grid_w + ds - 1) / ds;
@@ -161,9 +163,7 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
     tbv = tv;
   }
 
-  int* st = status ? status : &sc->status;
-  if (!status && cudaMemsetAsync(&sc->status, 0, sizeof(int), stream) != cudaSuccess)
-    return REGMEM_ERR_CUDA;
+  int* st = status;
   sampled_tokens_kernel<<<(nq + 255) / 256, 256, 0, stream>>>(sc->qidx, nq, fd->n_special,
                                                                fd->grid_w, ds, cols);
   if (cudaGetLastError() != cudaSuccess) return REGMEM_ERR_CUDA;

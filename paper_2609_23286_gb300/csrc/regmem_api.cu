@@ -15,10 +15,40 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "kernels.h"
 #include "regmem.h"
 
 using namespace regmem_dev;
+
+namespace {
+
+// One NVTX range per exported call, in the "regmem" domain, so that a
+// timeline (nsys, ncu's NVTX filters) shows which library call enqueued
+// which kernels.  With no tool attached a push/pop is a call through a null
+// function pointer check.
+nvtxDomainHandle_t nvtx_domain() {
+  static nvtxDomainHandle_t d = nvtxDomainCreateA("regmem");
+  return d;
+}
+struct NvtxRange {
+  explicit NvtxRange(const char* name) {
+    nvtxEventAttributes_t a = {};
+    a.version = NVTX_VERSION;
+    a.size = NVTX_EVENT_ATTRIB_STRUCT_SIZE;
+    a.messageType = NVTX_MESSAGE_TYPE_ASCII;
+    a.message.ascii = name;
+    nvtxDomainRangePushEx(nvtx_domain(), &a);
+  }
+  ~NvtxRange() { nvtxDomainRangePop(nvtx_domain()); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
+}  // namespace
+
+#define REGMEM_RANGE NvtxRange nvtx_range_(__func__)
 
 struct regmem {
   int layers = 0, heads = 0, head_dim = 0, budget = 0;
@@ -55,7 +85,7 @@ struct regmem {
   int* status_host = nullptr; // mapped pinned word written by kernels
   int* status_dev = nullptr;
 
-  // staging for the host-buffer entry point (allocated on first use)
+  // staging of the host-buffer entry points (allocated by regmem_set_frame)
   __nv_bfloat16* stQ = nullptr;
   __nv_bfloat16* stOut = nullptr;
   float* stSal = nullptr;
@@ -334,7 +364,43 @@ regmem_status regmem_create(regmem_t** out, int32_t layers, int32_t heads, int32
   return REGMEM_OK;
 }
 
+namespace {
+
+// Staging buffers, copy streams and events of the host-buffer entry points:
+// the six sets of regmem_attend_admit_host, and Q / out / saliency plus
+// per-layer K and V (kept until the layer's admit) of
+// regmem_attend_frame_host.  Made once, by regmem_set_frame, so that no
+// host-buffer call allocates (a cudaMalloc inside a stream of calls would
+// synchronise the device and stall the copies' overlap).
+regmem_status alloc_staging(regmem_t* h) {
+  const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
+  const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
+  RM_CUDA(h, cudaStreamCreateWithFlags(&h->cstream, cudaStreamNonBlocking));
+  RM_CUDA(h, cudaStreamCreateWithFlags(&h->dstream, cudaStreamNonBlocking));
+  for (auto& hs : h->hs) {
+    RM_CUDA(h, cudaMalloc(&hs.q, tbytes));
+    RM_CUDA(h, cudaMalloc(&hs.k, tbytes));
+    RM_CUDA(h, cudaMalloc(&hs.v, tbytes));
+    RM_CUDA(h, cudaMalloc(&hs.out, tbytes));
+    RM_CUDA(h, cudaMalloc(&hs.sal, sbytes));
+    RM_CUDA(h, cudaEventCreateWithFlags(&hs.h2d, cudaEventDisableTiming));
+    RM_CUDA(h, cudaEventCreateWithFlags(&hs.done, cudaEventDisableTiming));
+    RM_CUDA(h, cudaEventCreateWithFlags(&hs.d2h, cudaEventDisableTiming));
+  }
+  RM_CUDA(h, cudaMalloc(&h->stQ, tbytes));
+  RM_CUDA(h, cudaMalloc(&h->stOut, tbytes));
+  RM_CUDA(h, cudaMalloc(&h->stSal, sbytes));
+  for (int l = 0; l < h->layers; ++l) {
+    RM_CUDA(h, cudaMalloc(&h->stK[l], tbytes));
+    RM_CUDA(h, cudaMalloc(&h->stV[l], tbytes));
+  }
+  return REGMEM_OK;
+}
+
+}  // namespace
+
 regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
+  REGMEM_RANGE;
   if (!h || !fd) return REGMEM_ERR_ARG;
   if (h->frame_set) return fail(h, REGMEM_ERR_STATE, "frame geometry already set");
   const int ds = fd->ds == 0 ? 2 : fd->ds;
@@ -401,11 +467,14 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   h->max_frames = fd->max_frames;
   h->scale = fd->scale == 0.f ? 1.f / std::sqrt((float)h->head_dim) : fd->scale;
   h->cap = cap;
+  regmem_status s = alloc_staging(h);
+  if (s != REGMEM_OK) return s;
   h->frame_set = true;
   return REGMEM_OK;
 }
 
 regmem_status regmem_set_overlap(regmem_t* h, int32_t on) {
+  REGMEM_RANGE;
   if (!h || (on != 0 && on != 1)) return REGMEM_ERR_ARG;
   if (!on && h->frame_set && h->side_seq > h->covered_seq) {
     if (cudaSetDevice(h->device) != cudaSuccess)
@@ -418,6 +487,7 @@ regmem_status regmem_set_overlap(regmem_t* h, int32_t on) {
 }
 
 regmem_status regmem_join(regmem_t* h) {
+  REGMEM_RANGE;
   if (!h) return REGMEM_ERR_ARG;
   if (!h->frame_set || h->side_seq <= h->covered_seq) return REGMEM_OK;
   if (cudaSetDevice(h->device) != cudaSuccess)
@@ -531,6 +601,7 @@ regmem_status finish_side(regmem_t* h, int layer, cudaStream_t sst) {
 
 regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, const void* K,
                                   const void* V, void* out, float* saliency) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if ((s = check_tensors(h, Q, K, V, out, saliency)) != REGMEM_OK) return s;
@@ -551,6 +622,7 @@ regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, con
 regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, const void* K,
                                   const void* V, void* out, float* saliency, int32_t k,
                                   int32_t* idx_out) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if ((s = check_tensors(h, Q, K, V, out, saliency)) != REGMEM_OK) return s;
@@ -596,16 +668,6 @@ namespace {
 regmem_status stage_inputs(regmem_t* h, int32_t layer, const void* hostQ, const void* hostK,
                            const void* hostV) {
   const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
-  const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
-  if (!h->stQ) {
-    RM_CUDA(h, cudaMalloc(&h->stQ, tbytes));
-    RM_CUDA(h, cudaMalloc(&h->stOut, tbytes));
-    RM_CUDA(h, cudaMalloc(&h->stSal, sbytes));
-  }
-  if (!h->stK[layer]) {
-    RM_CUDA(h, cudaMalloc(&h->stK[layer], tbytes));
-    RM_CUDA(h, cudaMalloc(&h->stV[layer], tbytes));
-  }
   RM_CUDA(h, cudaMemcpyAsync(h->stQ, hostQ, tbytes, cudaMemcpyHostToDevice, h->stream));
   RM_CUDA(h, cudaMemcpyAsync(h->stK[layer], hostK, tbytes, cudaMemcpyHostToDevice, h->stream));
   RM_CUDA(h, cudaMemcpyAsync(h->stV[layer], hostV, tbytes, cudaMemcpyHostToDevice, h->stream));
@@ -625,6 +687,7 @@ regmem_status unstage_outputs(regmem_t* h, void* hostOut, float* hostSaliency) {
 regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* hostQ,
                                        const void* hostK, const void* hostV, void* hostOut,
                                        float* hostSaliency) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if (!hostQ || !hostK || !hostV || !hostOut || !hostSaliency)
@@ -638,31 +701,10 @@ regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, const void* h
   return unstage_outputs(h, hostOut, hostSaliency);
 }
 
-namespace {
-
-regmem_status host_set(regmem_t* h, regmem_t::HostSet& hs) {
-  const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
-  const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
-  if (!h->cstream) RM_CUDA(h, cudaStreamCreateWithFlags(&h->cstream, cudaStreamNonBlocking));
-  if (!h->dstream) RM_CUDA(h, cudaStreamCreateWithFlags(&h->dstream, cudaStreamNonBlocking));
-  if (!hs.q) {
-    RM_CUDA(h, cudaMalloc(&hs.q, tbytes));
-    RM_CUDA(h, cudaMalloc(&hs.k, tbytes));
-    RM_CUDA(h, cudaMalloc(&hs.v, tbytes));
-    RM_CUDA(h, cudaMalloc(&hs.out, tbytes));
-    RM_CUDA(h, cudaMalloc(&hs.sal, sbytes));
-    RM_CUDA(h, cudaEventCreateWithFlags(&hs.h2d, cudaEventDisableTiming));
-    RM_CUDA(h, cudaEventCreateWithFlags(&hs.done, cudaEventDisableTiming));
-    RM_CUDA(h, cudaEventCreateWithFlags(&hs.d2h, cudaEventDisableTiming));
-  }
-  return REGMEM_OK;
-}
-
-}  // namespace
-
 regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* hostQ,
                                        const void* hostK, const void* hostV, void* hostOut,
                                        float* hostSaliency, int32_t k) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if (!hostQ || !hostK || !hostV || !hostOut || !hostSaliency)
@@ -678,7 +720,6 @@ regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* h
   // streams are separate so that the next call's inputs need not wait for
   // this call's outputs: its copies overlap this call's kernels.
   regmem_t::HostSet& hs = h->hs[h->hs_next % regmem_t::kHostSets];
-  if ((s = host_set(h, hs)) != REGMEM_OK) return s;
   ++h->hs_next;
   const size_t tbytes = (size_t)h->N * h->heads * kHeadDim * 2;
   const size_t sbytes = (size_t)h->heads * h->N * sizeof(float);
@@ -708,6 +749,7 @@ regmem_status regmem_attend_admit_host(regmem_t* h, int32_t layer, const void* h
 }
 
 regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if (!h->pending[layer])
@@ -735,6 +777,7 @@ regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_o
 }
 
 regmem_status regmem_admit_shared(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if (!h->pending[layer])
@@ -755,6 +798,7 @@ regmem_status regmem_admit_shared(regmem_t* h, int32_t layer, int32_t k, int32_t
 
 regmem_status regmem_frame_attention(regmem_t* h, const void* Q, const void* K, const void* V,
                                      void* out) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, 0, false);
   if (s != REGMEM_OK) return s;
   if (!Q || !K || !V || !out) return fail(h, REGMEM_ERR_ARG, "null tensor pointer");
@@ -764,6 +808,7 @@ regmem_status regmem_frame_attention(regmem_t* h, const void* Q, const void* K, 
 }
 
 regmem_status regmem_reset(regmem_t* h) {
+  REGMEM_RANGE;
   if (!h) return REGMEM_ERR_ARG;
   if (h->frame_set && h->side_seq > h->covered_seq) {  // the new stream's writes follow the old side work
     if (cudaSetDevice(h->device) != cudaSuccess)
@@ -792,6 +837,7 @@ regmem_status regmem_capacity(const regmem_t* h, int64_t* rows) {
 }
 
 regmem_status regmem_export_bank(regmem_t* h, int32_t layer, void* hostK, void* hostV) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if (!hostK || !hostV) return fail(h, REGMEM_ERR_ARG, "null host pointer");
@@ -810,6 +856,7 @@ regmem_status regmem_export_bank(regmem_t* h, int32_t layer, void* hostK, void* 
 
 regmem_status regmem_import_bank(regmem_t* h, int32_t layer, const void* hostK, const void* hostV,
                                  int64_t len) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if (len < 0 || len > h->cap)
@@ -831,6 +878,7 @@ regmem_status regmem_import_bank(regmem_t* h, int32_t layer, const void* hostK, 
 }
 
 regmem_status regmem_copy_lse(regmem_t* h, float* dst) {
+  REGMEM_RANGE;
   regmem_status s = ready(h, 0, false);
   if (s != REGMEM_OK) return s;
   if (!dst) return fail(h, REGMEM_ERR_ARG, "null pointer");
@@ -840,6 +888,7 @@ regmem_status regmem_copy_lse(regmem_t* h, float* dst) {
 }
 
 regmem_status regmem_synchronize(regmem_t* h) {
+  REGMEM_RANGE;
   if (!h) return REGMEM_ERR_ARG;
   if (h->frame_set) {
     if (cudaSetDevice(h->device) != cudaSuccess)
@@ -854,6 +903,7 @@ regmem_status regmem_synchronize(regmem_t* h) {
 }
 
 regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention) {
+  REGMEM_RANGE;
   if (!h) return REGMEM_ERR_ARG;
   if (h->frame_set) {
     if (cudaSetDevice(h->device) != cudaSuccess)
@@ -875,6 +925,7 @@ regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention) {
 }
 
 regmem_status regmem_profile_read(regmem_t* h, regmem_profile* out) {
+  REGMEM_RANGE;
   if (!h || !out) return REGMEM_ERR_ARG;
   if (h->frame_set) {
     if (cudaSetDevice(h->device) != cudaSuccess)

@@ -226,7 +226,8 @@ def regmem_attend_frame_noalloc(n_special, grid_h, grid_w, heads, Q, K, V, bankK
                                 bank_rows, M, out, saliency, status=None, stream=None, ds=2,
                                 scale=0.0):
     """Handle-free attend step whose scratch is a fixed device array inside
-    the library (no device allocation)."""
+    the library (no device allocation).  `status` (a device int32, zeroed by
+    the caller) is required: the kernels record an expired wait there."""
     fd = FrameDesc(n_special + grid_h * grid_w, n_special, grid_h, grid_w, ds, 1, scale, 0)
     st = load().regmem_attend_frame_noalloc(ctypes.byref(fd), heads, _ptr(Q), _ptr(K), _ptr(V),
                                             _ptr(bankK), _ptr(bankV), bank_rows, M, _ptr(out),

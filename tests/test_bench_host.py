@@ -76,3 +76,39 @@ def test_attended_rows_follow_the_growth_law():
     assert bench.attended_rows(cfg, 1) == N                     # frame 1: no memory
     assert bench.attended_rows(cfg, 2) == 2 * N                 # anchor stored whole
     assert bench.attended_rows(cfg, 2000) - N == N + 1998 * 14  # |M_1999| = N + 1998 k
+
+
+def test_default_window_is_centred_on_the_mean_attended_length():
+    cfg = bench.CONFIGS["long"]
+    S0 = bench.default_start_frame(cfg["frames"], 20)
+    assert S0 == 991
+    frames = bench.window_frames(S0, 20)
+    assert frames[0] == 991 and frames[-1] == 1010
+    # the memory grows linearly (Eq. 6), so the mean over the stream is the
+    # middle frame's length; the window's mean is within one frame's k of it
+    whole = bench.mean_attended(cfg, range(1, cfg["frames"] + 1))
+    assert abs(bench.mean_attended(cfg, frames) - whole) <= cfg["k"]
+    assert bench.default_start_frame(100, 20) == 41
+    assert bench.default_start_frame(8, 6) == 2
+    assert bench.default_start_frame(2000, 0) == 1 and bench.default_start_frame(50, 50) == 1
+
+
+def test_reference_arm_line_uses_the_same_frames_and_config():
+    """The oracle arm runs on CPU: its config equals the GPU arm's config for
+    the same command line, and its steps sample the timed window."""
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--config", "tiny",
+                          "--steps", "3", "--warmup", "1"], cwd=root, capture_output=True,
+                         text=True, timeout=300)
+    assert out.returncode == 0, out.stderr[-2000:]
+    d = json.loads(out.stdout.strip().splitlines()[-1])
+    cfg = bench.CONFIGS["tiny"]
+    S0 = bench.default_start_frame(cfg["frames"], 3)
+    assert d["impl"] == "reference" and d["steps"] == 3 and d["warmup"] == 1
+    assert d["config"] == json.loads(json.dumps(bench.bench_config(cfg, "tiny", S0, 3, 1)))
+    assert d["config"]["first_frame"] == S0 == 4  # frames 4-6 of 8, centred on frame 5
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+    assert d["value"] > 0 and d["unit"] == bench.UNIT and d["metric"] == bench.METRIC

@@ -9,7 +9,8 @@ import pytest
 import torch
 
 import oracle as orc
-from helpers import (Stream, check_indices, check_lse, check_o, check_saliency, to64)
+from helpers import (Stream, check_indices, check_lse, check_o, check_saliency, o_abs_frame,
+                     to64)
 from paper_2609_23286_gb300 import regmem
 
 pytestmark = pytest.mark.gpu
@@ -32,9 +33,11 @@ def run_stream(L, H, ns, gh, gw, k, frames, seed, ds=2, check_every=1, fused=Fal
                     out, sal, lse = st.attend(layer, q, kk_, v)
                     idx = st.admit(layer, k)
                 torch.cuda.synchronize()
+                oa = o_abs_frame(to64(q), to64(kk_), to64(v), ref.bank_k[layer],
+                                 ref.bank_v[layer], ref.scale)
                 r = ref.attend(layer, to64(q), to64(kk_), to64(v))
                 if t % check_every == 0 or t <= 2:
-                    check_o(out, r["O"], f"t={t} l={layer}")
+                    check_o(out, r["O"], f"t={t} l={layer}", o_abs=oa)
                     check_lse(lse, r["LSE"], f"t={t} l={layer}")
                     check_saliency(sal, r["S"], f"t={t} l={layer}")
                 if ref.memory_len(layer) == 0:
@@ -105,10 +108,12 @@ def test_teacher_forced_bank_lengths(M):
         out, sal, lse = st.attend(0, q, k, v)
         idx = st.admit(0, 14)
         torch.cuda.synchronize()
-        ref = orc.attend_frame(to64(q), to64(k), to64(v), [bk[h].double().numpy() for h in range(H)],
-                               [bv[h].double().numpy() for h in range(H)], 1 / 8,
+        bk64 = [bk[h].double().numpy() for h in range(H)]
+        bv64 = [bv[h].double().numpy() for h in range(H)]
+        ref = orc.attend_frame(to64(q), to64(k), to64(v), bk64, bv64, 1 / 8,
                                orc.sampled_query_tokens(ns, gh, gw, 2))
-        check_o(out, ref["O"], f"M={M}")
+        oa = o_abs_frame(to64(q), to64(k), to64(v), bk64, bv64, 1 / 8)
+        check_o(out, ref["O"], f"M={M}", o_abs=oa)
         check_lse(lse, ref["LSE"], f"M={M}")
         check_saliency(sal, ref["S"], f"M={M}")
         check_indices(idx.cpu().numpy(), to64(sal), ref["S"], ns, 14, 361)
@@ -144,10 +149,12 @@ def test_split_units_across_many_ctas(H, ns, gh, gw, M):
         q, k, v = st.inputs(0, 3)
         out, sal, lse = st.attend(0, q, k, v)
         torch.cuda.synchronize()
-        ref = orc.attend_frame(to64(q), to64(k), to64(v), [bk[h].double().numpy() for h in range(H)],
-                               [bv[h].double().numpy() for h in range(H)], 1 / 8,
+        bk64 = [bk[h].double().numpy() for h in range(H)]
+        bv64 = [bv[h].double().numpy() for h in range(H)]
+        ref = orc.attend_frame(to64(q), to64(k), to64(v), bk64, bv64, 1 / 8,
                                orc.sampled_query_tokens(ns, gh, gw, 2))
-        check_o(out, ref["O"], f"H={H} N={N} M={M}")
+        oa = o_abs_frame(to64(q), to64(k), to64(v), bk64, bv64, 1 / 8)
+        check_o(out, ref["O"], f"H={H} N={N} M={M}", o_abs=oa)
         check_lse(lse, ref["LSE"], f"H={H} N={N} M={M}")
         check_saliency(sal, ref["S"], f"H={H} N={N} M={M}")
     finally:
@@ -176,13 +183,15 @@ def test_running_max_renewed_by_large_later_logits():
         q, k, v = st.inputs(0, 3)
         out, sal, lse = st.attend(0, q, k, v)
         torch.cuda.synchronize()
-        ref = orc.attend_frame(to64(q), to64(k), to64(v), [bk[h].double().numpy() for h in range(H)],
-                               [bv[h].double().numpy() for h in range(H)], 1 / 8,
+        bk64 = [bk[h].double().numpy() for h in range(H)]
+        bv64 = [bv[h].double().numpy() for h in range(H)]
+        ref = orc.attend_frame(to64(q), to64(k), to64(v), bk64, bv64, 1 / 8,
                                orc.sampled_query_tokens(ns, gh, gw, 2))
+        oa = o_abs_frame(to64(q), to64(k), to64(v), bk64, bv64, 1 / 8)
         # the case is only meaningful if many rows' logits outgrow the first tiles' by far
         z_big = to64(q)[:, 0, :].sum(axis=1) * 50.0 / 8.0
         assert (z_big * 1.4426950408889634 > 64 + 5).sum() > 50
-        check_o(out, ref["O"], "renewed running max")
+        check_o(out, ref["O"], "renewed running max", o_abs=oa)
         check_lse(lse, ref["LSE"], "renewed running max")
         check_saliency(sal, ref["S"], "renewed running max")
     finally:
@@ -212,7 +221,8 @@ def test_long_bank_sampled_rows():
             kc = np.concatenate([bk[h].double().numpy(), k64[:, h]])
             vc = np.concatenate([bv[h].double().numpy(), v64[:, h]])
             o_r, l_r, _, _ = orc.attend_head(q64[rows, h], kc, vc, 1 / 8)
-            check_o(out[rows, h], o_r, f"h={h}")
+            o_a, _, _, _ = orc.attend_head(q64[rows, h], kc, np.abs(vc), 1 / 8)
+            check_o(out[rows, h], o_r, f"h={h}", o_abs=o_a)
             check_lse(lse[h, rows], l_r, f"h={h}")
             _, l_s, z_s, _ = orc.attend_head(q64[qi, h], kc, vc, 1 / 8)
             s_r = orc.saliency_lse(z_s, l_s, M, list(range(len(qi))))
@@ -234,7 +244,9 @@ def test_frame_attention_matches_sdpa_oracle():
         torch.cuda.synchronize()
         ref = orc.attend_frame(to64(q), to64(k), to64(v), [np.zeros((0, 64))] * H,
                                [np.zeros((0, 64))] * H, 1 / 8, [0])
-        check_o(out, ref["O"], "frame attention")
+        oa = o_abs_frame(to64(q), to64(k), to64(v), [np.zeros((0, 64))] * H,
+                         [np.zeros((0, 64))] * H, 1 / 8)
+        check_o(out, ref["O"], "frame attention", o_abs=oa)
         assert st.rm.memory_len(0) == 0
     finally:
         st.close()
@@ -276,6 +288,45 @@ def test_host_buffer_entry_point_matches_device_path():
     finally:
         a.close()
         b.close()
+
+
+def test_host_entry_points_allocate_nothing_after_set_frame():
+    """regmem_set_frame makes every staging buffer, copy stream and event of
+    the host-buffer calls: once the kernels are loaded (two warm-up frames),
+    a run of host calls that cycles through all six staging sets of
+    regmem_attend_admit_host, plus the two-call host form, leaves the
+    device's free memory (cudaMemGetInfo) unchanged."""
+    H, ns, gh, gw = 16, 5, 37, 37
+    N = ns + gh * gw
+    st = Stream(2, H, ns, gh, gw, budget=14, max_frames=16, seed=16)
+    try:
+        frames = [tuple(x.cpu().pin_memory() for x in st.inputs(l, t)) for t in range(1, 5)
+                  for l in range(2)]
+        ho = torch.empty(N, H, 64, dtype=torch.bfloat16).pin_memory()
+        hs = torch.empty(H, N, dtype=torch.float32).pin_memory()
+
+        def host_frame(i):
+            for l in range(2):
+                q, k, v = frames[(2 * i + l) % len(frames)]
+                st.rm.attend_admit_host(l, q, k, v, ho, hs, 14)
+
+        for i in range(2):  # anchor and first admitted frame: every kernel loaded
+            host_frame(i)
+        q, k, v = frames[0]
+        st.rm.attend_frame_host(0, q, k, v, ho, hs)
+        st.rm.admit(0, 14)
+        st.rm.synchronize()
+        torch.cuda.synchronize()
+        free0 = torch.cuda.mem_get_info()[0]
+        for i in range(2, 9):  # 14 calls: every staging set used twice or more
+            host_frame(i)
+        st.rm.attend_frame_host(1, q, k, v, ho, hs)
+        st.rm.admit(1, 14)
+        st.rm.synchronize()
+        torch.cuda.synchronize()
+        assert torch.cuda.mem_get_info()[0] == free0
+    finally:
+        st.close()
 
 
 def test_deterministic_repeat():

@@ -52,8 +52,19 @@ def test_noalloc_matches_handle_path_on_two_calls():
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch():
+    z = torch.zeros(16, dtype=torch.bfloat16, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
     with pytest.raises(regmem.RegmemError) as e:
-        z = torch.zeros(16, dtype=torch.bfloat16, device="cuda")
         # 64 heads x 4101 tokens > 262144 LSE rows held by the scratch
-        regmem.regmem_attend_frame_noalloc(5, 64, 64, 64, z, z, z, None, None, 0, 0, z, z)
+        regmem.regmem_attend_frame_noalloc(5, 64, 64, 64, z, z, z, None, None, 0, 0, z, z,
+                                           status=status)
     assert e.value.status == regmem.ERR_UNSUPPORTED
+
+
+def test_noalloc_requires_a_status_word():
+    """Without a handle no later call could report an expired device wait, so
+    the caller's status word is mandatory."""
+    z = torch.zeros(16, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(regmem.RegmemError) as e:
+        regmem.regmem_attend_frame_noalloc(5, 2, 2, 2, z, z, z, None, None, 0, 0, z, z)
+    assert e.value.status == regmem.ERR_ARG
