@@ -50,14 +50,15 @@
 // (S(j) read into registers), p_ready (P(j) stored), o_done (P V(j) done);
 // plus the K/V ring's full/empty barriers (the empty ones take one arrival
 // from each issuer) and Q full/empty.  On GB300 every mbarrier hand-off costs
-// a few hundred cycles of latency, even on a phase that has already
-// completed, so the design keeps them off the critical chain where it can:
-// the softmax releases S as soon as it holds S(j) in registers, and the
-// Q K^T issuer computes S(j+1) while the softmax works on tile j; P is
-// single-buffered, so the softmax waits for P V(j-1) before storing P(j):
-// the tile's P V issuer, idle until the next p_ready anyway, waits for each
-// P V to complete and publishes the count in a shared word, which the
-// softmax checks with one shared load instead of an mbarrier wait.
+// a few hundred cycles of latency, so the design keeps them off the critical
+// chain where it can: the softmax releases S as soon as it holds S(j) in
+// registers, and the Q K^T issuer computes S(j+1) while the softmax works on
+// tile j; P is single-buffered, so the softmax waits for P V(j-1) (its
+// o_done phase) before storing P(j).  The P V issuer never waits for its
+// MMAs to complete: it commits each P V to o_done and moves on to the next
+// p_ready, so P V(j) is issued as soon as P(j) is stored (measured 1 %
+// shorter launches than an issuer that waited for each P V and published
+// its completion in a shared word).
 // With separate issuers for Q K^T and for each tile's P V, a Q K^T is never
 // queued behind the issue of a P V in the same thread (an MMA issue blocks
 // while the tensor core is busy), and one tile's P V never waits for the
@@ -93,7 +94,6 @@ constexpr uint32_t TM_S0 = 0, TM_S1 = 128, TM_P0 = 256, TM_P1 = 320, TM_O0 = 384
 constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s: a hung pipeline gives up
 constexpr uint64_t DRAIN_NS = 200000000ull;   // 0.2 s for draining on abort
 constexpr float RESCALE_LOG2 = 8.0f;
-constexpr uint32_t FLAG_ABORT = 0x7fffffffu;  // an issuer gave up
 constexpr uint32_t IDESC_QK = idesc_bf16_f32(128, 128, false, false);
 constexpr uint32_t IDESC_PV = idesc_bf16_f32(128, 64, false, true);
 
@@ -108,9 +108,6 @@ struct Smem {
   uint32_t tmem_base;
   int abort_flag;
   int never;  // always 0: abort word for waits that must not be cut short
-  // P V completions per query tile, published by its P V issuer (the softmax
-  // checks this word instead of the o_done mbarrier)
-  uint32_t flag_o[2];
 };
 // The dynamic shared window is requested 1 KB aligned (128-byte swizzle
 // atoms need it) and checked at run time.
@@ -174,7 +171,6 @@ __global__ void __launch_bounds__(THREADS, 1)
   if (tid == 0) {
     sm.abort_flag = 0;
     sm.never = 0;
-    sm.flag_o[0] = sm.flag_o[1] = 0;
     mbar_init(smem_addr(&sm.q_full), 1);
     mbar_init(smem_addr(&sm.q_empty), 1);
     for (int s = 0; s < STAGES; ++s) {
@@ -311,19 +307,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             ++ph1;
           }
         } else if (tpv == 0 || pc.ut.has1) {
-          // P V(j) of the query tile goes out once P(j) is stored; the stage
-          // is released when it completes (the last read of its V)
+          // P V(j) of the query tile goes out once P(j) is stored; its
+          // completion releases P (o_done, waited by the softmax) and the
+          // stage (the last read of its V).  The issuer does not wait for it.
           const uint32_t b_pready = smem_addr(&sm.p_ready[tpv]), b_odone = smem_addr(&sm.o_done[tpv]);
-          const uint32_t f_pub = smem_addr(&sm.flag_o[tpv]);
           const uint32_t d_o = tmem + (tpv ? TM_O1 : TM_O0), d_p = tmem + (tpv ? TM_P1 : TM_P0);
           for (int jj = 0; jj < n && ok; ++jj) {
             const int st = use_of(jj, tpv) % STAGES;
             ok = mbar_wait(b_pready, ph0 & 1, abort_flag, WAIT_NS);
             ++ph0;
-            if (!ok) {
-              st_release_shared(f_pub, FLAG_ABORT);
-              break;
-            }
+            if (!ok) break;
             tc_fence_after();
             const uint32_t vaddr = smem_addr(sm.v[st]);
 #pragma unroll
@@ -332,12 +325,6 @@ __global__ void __launch_bounds__(THREADS, 1)
                      (jj == 0 && kk == 0) ? 0u : 1u);
             mma_commit(b_odone);
             mma_commit(smem_addr(&sm.kv_empty[st]));
-            // publish P V(jj) once complete (the softmax stores P(jj+1)
-            // after it); nothing else waits on this thread until p_ready
-            const bool done = mbar_wait(b_odone, ph1 & 1, abort_flag, WAIT_NS);
-            ++ph1;
-            ok = done;
-            st_release_shared(f_pub, done ? ph1 : FLAG_ABORT);
             if (ok && pc.kvs == 2) {
               // the other head's stage of this key tile: this issuer's release
               // of it (an arrival only after that use's load has landed)
@@ -375,31 +362,13 @@ __global__ void __launch_bounds__(THREADS, 1)
     const uint32_t b_sfree = smem_addr(&sm.s_free[t]), b_odone = smem_addr(&sm.o_done[t]);
     const uint32_t tm_p = tmem + lane_off + (t ? TM_P1 : TM_P0);
     const float c = p.scale_log2;
-    const uint32_t f_o = smem_addr(&sm.flag_o[t]);
     uint32_t s_phase = 0, o_phase = 0;  // s_full parity, P V completions consumed
     bool stop = false;
-    // Waits until the issuer has published `target` completions (bounded:
-    // gives up on the abort word or after WAIT_NS).  One shared load per
-    // check; the load is warp-wide, so the result is uniform across the warp.
+    // Bounded wait for a barrier phase (gives up on the abort word or after
+    // WAIT_NS); a warp stops as a whole if any of its lanes gave up.
     auto wait_phase = [&](uint32_t bar, uint32_t parity) -> bool {
       const bool ok = mbar_wait(bar, parity, abort_flag, WAIT_NS);
       if (__any_sync(0xffffffffu, !ok)) return false;
-      tc_fence_after();
-      return true;
-    };
-    auto wait_flag = [&](uint32_t flag, uint32_t target) -> bool {
-      uint32_t v = ld_acquire_shared(flag);
-      if (v < target) {
-        const uint64_t t0 = globaltimer_ns();
-        for (int i = 1; v < target; ++i) {
-          v = ld_acquire_shared(flag);
-          if ((i & 255) == 0 && v < target && (*abort_flag || globaltimer_ns() - t0 > WAIT_NS)) {
-            *abort_flag = 1;
-            return false;
-          }
-        }
-      }
-      if (v == FLAG_ABORT) return false;
       tc_fence_after();
       return true;
     };
@@ -472,8 +441,9 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
         }
         if (jj > 0) {
-          // P V(j-1) has read P and added into O
-          if (!wait_flag(f_o, ++o_phase)) {
+          // P V(j-1) has read P and added into O (at most one P V of this
+          // tile is outstanding here, so the parity is unambiguous)
+          if (!wait_phase(b_odone, (o_phase++) & 1)) {
             stop = true;
             break;
           }
@@ -503,7 +473,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       if (stop) break;
       // -------------------------------------------------------------- epilogue
-      if (!wait_flag(f_o, ++o_phase)) {  // the last tile's P V
+      if (!wait_phase(b_odone, (o_phase++) & 1)) {  // the last tile's P V
         stop = true;
         break;
       }

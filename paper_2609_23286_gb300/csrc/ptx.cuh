@@ -96,17 +96,6 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 }
 
 
-// CTA-scope release store / acquire load of a shared-memory word (a hand-off
-// between warps of one CTA that costs one shared-memory access to check).
-__device__ __forceinline__ void st_release_shared(uint32_t addr, uint32_t v) {
-  asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
-__device__ __forceinline__ uint32_t ld_acquire_shared(uint32_t addr) {
-  uint32_t v;
-  asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
-  return v;
-}
-
 // ---------------------------------------------------------------------------
 // mbarrier
 // ---------------------------------------------------------------------------
@@ -146,14 +135,31 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking test of the phase with the given parity.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 // Waits for the phase of `bar` with the given parity to complete.  Gives up
 // when *abort is set by another thread, or after `timeout_ns` of wall time
 // (then sets *abort itself).  Returns true only on completion.
-// The common case -- the phase completes within a few hundred polls -- never
-// touches the timer; after that the abort word and the timer are checked
-// once every 64 polls.
+// A phase that has already completed -- the common case on the pipeline's
+// hand-offs -- is caught by one non-blocking test: on GB300 that is cheaper
+// than try_wait, which costs a few hundred cycles even on a completed phase
+// (measured: the attention launch 2.5 % shorter).  Spinning on the test
+// instead of try_wait measured slower (it takes issue slots from the warps
+// doing the work).  The next polls never touch the timer; after a few
+// hundred, the abort word and the timer are checked once every 64 polls.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort,
                                           uint64_t timeout_ns) {
+  if (mbar_test_wait(bar, parity)) return true;
 #pragma unroll 1
   for (int i = 0; i < 512; ++i)
     if (mbar_try_wait(bar, parity)) return true;
