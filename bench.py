@@ -354,6 +354,36 @@ def _oracle_entry(cfg_json, what, steps, warmup, S0, K):
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+def parse_cpulist(text):
+    cpus = set()
+    for part in text.strip().split(","):
+        if not part:
+            continue
+        lo, _, hi = part.partition("-")
+        cpus.update(range(int(lo), int(hi or lo) + 1))
+    return cpus
+
+
+def bind_near_gpu(index):
+    """Restricts this process to the CPUs attached to GPU `index` (its NUMA
+    node, from sysfs), so that host buffers pinned afterwards are placed in
+    the memory nearest the GPU and its copy engines do not cross the
+    socket link.  Returns what was done, or None where sysfs does not say."""
+    import torch
+    try:
+        pr = torch.cuda.get_device_properties(index)
+        bus = f"{pr.pci_domain_id:04x}:{pr.pci_bus_id:02x}:{pr.pci_device_id:02x}.0"
+        base = f"/sys/bus/pci/devices/{bus}"
+        cpus = parse_cpulist(open(f"{base}/local_cpulist").read()) & os.sched_getaffinity(0)
+        node = open(f"{base}/numa_node").read().strip()
+    except (AttributeError, OSError, ValueError):
+        return None
+    if not cpus:
+        return None
+    os.sched_setaffinity(0, cpus)
+    return {"pci": bus, "numa_node": int(node), "cpus": len(cpus)}
+
+
 def make_pool(cfg, P, seed, device):
     import torch
     from paper_2609_23286_gb300 import synth
@@ -439,6 +469,10 @@ def gpu_arm(args, cfg, cfg_name):
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = run_oracle_subprocess(cfg, "baseline", S0=S0, K=K)
+
+    # after the oracle baseline (which uses every core): this process keeps
+    # to the GPU's own CPUs, where its pinned host buffers are then placed
+    placement = bind_near_gpu(local_rank)
 
     P = min(args.pool, max(K, W, 1))
     pool = make_pool(cfg, P, seed, dev)
@@ -595,6 +629,7 @@ def gpu_arm(args, cfg, cfg_name):
             "overlap": ("saliency + admission on a side stream" if args.overlap
                         else "all kernels on one stream"),
             "timed_region_ms": round(ms, 3),
+            "host_placement": placement,
         },
         "tflops_attention_path": round(flops_total / (ms / 1e3) / 1e12 * world, 2),
         "roofline": {

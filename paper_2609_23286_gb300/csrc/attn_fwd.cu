@@ -12,8 +12,9 @@
 // Work split (stream-K over the key dimension): a unit is a pair of 128-row
 // query tiles -- two consecutive tiles of one head, or the last tiles of two
 // heads when a head has an odd number of them (unit_tiles) -- and the
-// (unit, key tile) space is cut into
-// `grid` contiguous equal ranges, one per CTA (one CTA per SM).  A unit whose
+// (unit, key tile) space is cut into `grid` contiguous ranges of about equal
+// estimated cost, one per CTA (one CTA per SM; attn_split_bounds: a frame
+// tile and the start of a unit cost more than a bank tile).  A unit whose
 // key tiles all fall in one CTA is finished there (O in bf16 and LSE written
 // directly).  A unit cut between CTAs leaves one normalised fp32 partial
 // (O_p, LSE_p) per piece, in a slot of the CTA that computed it (its first or
@@ -115,6 +116,7 @@ constexpr size_t SMEM_BYTES = (sizeof(Smem) + 127) & ~size_t(127);
 static_assert(SMEM_BYTES <= 232448, "more dynamic shared memory than a CTA can have (227 KB)");
 
 struct Params {
+  SplitBounds bnd;  // this launch's split: CTA b takes tiles [bnd.x[b], bnd.x[b + 1])
   int N, H, M;
   int nb, nkv, nqt;
   long long total;
@@ -128,8 +130,6 @@ struct Params {
   unsigned long long* clk_end;
 };
 
-using split::cta_of;
-using split::range_begin;
 
 __device__ __forceinline__ int tile_valid(const Params& p, int j) {
   return j < p.nb ? min(BN, p.M - j * BN) : min(BN, p.N - (j - p.nb) * BN);
@@ -166,7 +166,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   volatile int* never = &sm.never;
 
   const int G = gridDim.x, b = blockIdx.x;
-  const long long x_begin = range_begin(b, G, p.total), x_end = range_begin(b + 1, G, p.total);
+  const long long x_begin = p.bnd.x[b], x_end = p.bnd.x[b + 1];
 
   if (tid == 0) {
     sm.abort_flag = 0;
@@ -556,6 +556,12 @@ __global__ void __launch_bounds__(CMB_THREADS, 2)
 
 Params make_params(const AttnArgs& a) {
   Params p;
+  {
+    const int nb = (a.M + BN - 1) / BN, nf = (a.N + BN - 1) / BN;
+    const long long units = attn_units((a.N + BM - 1) / BM, a.H);
+    const long long total = units * (nb + nf);
+    attn_split_bounds(p.bnd, units, nb, nf, (int)(a.grid < total ? a.grid : total));
+  }
   p.N = a.N;
   p.H = a.H;
   p.M = a.M;
@@ -580,6 +586,7 @@ Params make_params(const AttnArgs& a) {
 SplitLayout attn_split_layout(const AttnArgs& a) {
   const Params p = make_params(a);
   SplitLayout l;
+  l.bnd = p.bnd;
   l.total = p.total;
   l.G = a.grid;
   l.nkv = p.nkv;

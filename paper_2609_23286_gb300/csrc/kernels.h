@@ -35,11 +35,48 @@ constexpr int kTile = 128;      // query rows / key rows per tile
 constexpr int kStatusTimeout = 1;    // a bounded wait expired
 constexpr int kStatusSmemAlign = 2;  // dynamic shared memory not 1 KB aligned
 
-// Attention over [bank rows ; frame rows] for every (head, 128-row query tile).
-// The attention's stream-K split, as the merge of split units needs it
-// (split.cuh): CTA b takes tiles [b total / G, (b + 1) total / G) of the
-// (unit, key tile) sequence.
+// Largest attention grid: the merge of split units lists at most this many
+// pieces per unit.
+constexpr int kAttnMaxGrid = 256;
+
+// The attention's stream-K split: CTA b takes key tiles [x[b], x[b + 1]) of
+// the (unit, key tile) sequence.  The cuts equalise an estimated cost, not
+// the tile count: a frame tile (the frame's own K/V, gathered from the
+// token-major frame tensor, the last one ragged) costs more than a bank
+// tile, and every unit a CTA starts costs a pipeline drain and refill.  The
+// weights are per-CTA timings of the kernel at 16.7k keys regressed on
+// these counts (a unit start ~1.7 tiles, a frame tile ~1.08).
+constexpr int kCostBankTile = 100, kCostFrameTile = 108, kCostUnitStart = 170;
+struct SplitBounds {
+  long long x[kAttnMaxGrid + 1];
+};
+// Cuts `units` units of nb bank tiles followed by nf frame tiles into G
+// ranges of about equal cost (1 <= G <= units * (nb + nf)): strictly
+// increasing, x[0] = 0, x[G] = units * (nb + nf).
+inline void attn_split_bounds(SplitBounds& sb, long long units, int nb, int nf, int G) {
+  const long long nkv = nb + nf, total = units * nkv;
+  const long long wu = kCostUnitStart + (long long)kCostBankTile * nb + (long long)kCostFrameTile * nf;
+  const long long wt = units * wu;
+  for (int b = 0; b <= G; ++b) {
+    const long long target = wt / G * b + (wt % G) * b / G;  // floor(wt b / G) without overflow
+    const long long u = target / wu;
+    long long r = target - u * wu - kCostUnitStart, j;
+    if (r <= 0) j = 0;
+    else if (r < (long long)kCostBankTile * nb) j = (r + kCostBankTile / 2) / kCostBankTile;
+    else j = nb + (r - (long long)kCostBankTile * nb + kCostFrameTile / 2) / kCostFrameTile;
+    sb.x[b] = u * nkv + (j < nkv ? j : nkv);
+  }
+  sb.x[0] = 0;
+  sb.x[G] = total;
+  for (int b = 1; b < G; ++b)  // every CTA at least one tile
+    if (sb.x[b] <= sb.x[b - 1]) sb.x[b] = sb.x[b - 1] + 1;
+  for (int b = G - 1; b > 0; --b)
+    if (sb.x[b] > total - (G - b)) sb.x[b] = total - (G - b);
+}
+
+// The split as the merge of split units needs it (split.cuh).
 struct SplitLayout {
+  SplitBounds bnd;
   long long total;        // units * nkv
   int G;                  // attention CTAs
   int nkv;                // key tiles per unit
@@ -118,9 +155,6 @@ struct AttnPlan {
 };
 AttnPlan attn_plan(int N, int H, int M);
 
-// Largest attention grid: the merge of split units lists at most this many
-// pieces per unit.
-constexpr int kAttnMaxGrid = 256;
 // Scratch sizes for a given grid.
 inline size_t attn_part_o_elems(int grid) { return (size_t)grid * 2 * kUnitRows * kHeadDim; }
 inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kUnitRows; }

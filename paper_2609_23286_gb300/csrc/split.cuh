@@ -2,7 +2,8 @@
 //
 // The (unit, key tile) sequence -- a unit is a pair of 128-row query tiles
 // (unit_tiles), run over every key tile of [bank ; frame] -- is cut into G
-// contiguous equal ranges, CTA b taking [b T / G, (b + 1) T / G).  A unit cut
+// contiguous ranges of about equal cost (attn_split_bounds), CTA b taking
+// [x[b], x[b + 1]).  A unit cut
 // by a CTA boundary leaves, from each CTA that holds part of it, one
 // normalised partial per query row, (O_p, LSE_p), in the CTA's slot 0 (the
 // unit is the CTA's first piece) or 1 (its last piece), O_p in bf16 and LSE_p
@@ -30,16 +31,19 @@ constexpr int kPrefetch = 2;            // pieces whose loads are issued togethe
 
 using Layout = SplitLayout;
 
-__host__ __device__ __forceinline__ long long range_begin(int b, int G, long long T) {
-  return (long long)b * T / G;
+__host__ __device__ __forceinline__ long long range_begin(const SplitBounds& sb, int b) {
+  return sb.x[b];
 }
 
-// CTA whose range contains tile x.
-__device__ __forceinline__ int cta_of(long long x, int G, long long T) {
-  long long b = x * G / T;
-  while (b + 1 < G && range_begin((int)b + 1, G, T) <= x) ++b;
-  while (b > 0 && range_begin((int)b, G, T) > x) --b;
-  return (int)b;
+// CTA whose range contains tile x (binary search of the cuts).
+__host__ __device__ __forceinline__ int cta_of(const SplitBounds& sb, int G, long long x) {
+  int lo = 0, hi = G - 1;  // sb.x[lo] <= x < sb.x[hi + 1]
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (sb.x[mid] <= x) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
 }
 
 // The CTAs holding a split unit: b_lo .. b_hi, and the slot of b_lo's piece
@@ -141,10 +145,10 @@ struct Job {
 // Whether job j merges anything (host and device).
 __host__ __device__ inline bool job_live(const Layout& s, int j) {
   const int bnd = j / 2 + 1;
-  const long long xb = range_begin(bnd, s.G, s.total);
+  const long long xb = range_begin(s.bnd, bnd);
   const int u = (int)(xb / s.nkv);
   const long long x0 = (long long)u * s.nkv;
-  if (xb == x0 || range_begin(bnd - 1, s.G, s.total) > x0) return false;
+  if (xb == x0 || range_begin(s.bnd, bnd - 1) > x0) return false;
   return (j & 1) == 0 || unit_tiles(u, s.nqt, s.H).has1;
 }
 __device__ __forceinline__ Job prepare_job(const Layout& s, int j) {
@@ -153,12 +157,12 @@ __device__ __forceinline__ Job prepare_job(const Layout& s, int j) {
   jb.t = j & 1;
   if (j < 0 || !job_live(s, j)) return jb;
   const int bnd = j / 2 + 1;
-  const long long x0 = range_begin(bnd, s.G, s.total) / s.nkv * s.nkv;
+  const long long x0 = range_begin(s.bnd, bnd) / s.nkv * s.nkv;
   const int u = (int)(x0 / s.nkv);
   jb.u = u;
   jb.pc.b_lo = bnd - 1;  // the CTA holding the unit's first tile
-  jb.pc.b_hi = cta_of(x0 + s.nkv - 1, s.G, s.total);
-  jb.pc.which_lo = range_begin(jb.pc.b_lo, s.G, s.total) == x0 ? 0 : 1;
+  jb.pc.b_hi = cta_of(s.bnd, s.G, x0 + s.nkv - 1);
+  jb.pc.which_lo = range_begin(s.bnd, jb.pc.b_lo) == x0 ? 0 : 1;
   return jb;
 }
 template <int NT>

@@ -112,3 +112,9 @@ def test_reference_arm_line_uses_the_same_frames_and_config():
     assert d["config"]["first_frame"] == S0 == 4  # frames 4-6 of 8, centred on frame 5
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
     assert d["value"] > 0 and d["unit"] == bench.UNIT and d["metric"] == bench.METRIC
+
+
+def test_cpulist_parser():
+    assert bench.parse_cpulist("0-3,8,10-11\n") == {0, 1, 2, 3, 8, 10, 11}
+    assert bench.parse_cpulist("72-143") == set(range(72, 144))
+    assert bench.parse_cpulist("") == set()
