@@ -284,6 +284,22 @@ REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_frame_desc* fd
                                                      float* saliency, int32_t* status,
                                                      void* stream);
 
+/* Failure-detection hook, for tests.  The paper has no counterpart.
+ * wait_limit_us sets the limit of every bounded wait inside the attention
+ * kernel for this handle's later launches (default 2,000,000 us = 2 s;
+ * 1 <= wait_limit_us <= 60 s).  skip_kv_load >= 0 arms a one-shot fault for
+ * the NEXT attention launch only: the first CTA's TMA producer does not
+ * issue its skip_kv_load-th K/V tile load (CTA-local index, from 0), so
+ * nothing ever lands in that ring stage; the consumers' bounded waits on it
+ * run out after the limit, every role of that CTA stops, drains the copies
+ * and MMAs it has issued, frees its tensor memory and sets the timeout bit
+ * of the handle's status word.  The GPU context stays usable: the next call
+ * (and regmem_synchronize) returns REGMEM_ERR_TIMEOUT and the handle must
+ * then be destroyed.  The index must be below the number of K/V loads of the
+ * first CTA, else nothing is skipped.  skip_kv_load = -1 disarms.  Nothing
+ * is enqueued.  ERR_ARG on out-of-range values. */
+REGMEM_API regmem_status regmem_debug_set(regmem_t* h, int64_t wait_limit_us, int32_t skip_kv_load);
+
 /* Launch counters and kernel timing, for measurement tools.
  * Counters cover every kernel this handle launched since the last
  * regmem_profile_enable.  When time_attention is set, CUDA events are

@@ -92,7 +92,6 @@ constexpr uint32_t REGS_CTRL = 56, REGS_SOFTMAX = 224;
 static_assert(128 * REGS_CTRL + 256 * REGS_SOFTMAX <= THREADS * 168, "register split");
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t TM_S0 = 0, TM_S1 = 128, TM_P0 = 256, TM_P1 = 320, TM_O0 = 384, TM_O1 = 448;
-constexpr uint64_t WAIT_NS = 2000000000ull;   // 2 s: a hung pipeline gives up
 constexpr uint64_t DRAIN_NS = 200000000ull;   // 0.2 s for draining on abort
 constexpr float RESCALE_LOG2 = 8.0f;
 constexpr uint32_t IDESC_QK = idesc_bf16_f32(128, 128, false, false);
@@ -128,6 +127,8 @@ struct Params {
   int* status;
   unsigned long long* clk_start;  // launch clock (AttnArgs) or nullptr
   unsigned long long* clk_end;
+  unsigned long long wait_ns;     // limit of every bounded wait (AttnArgs)
+  int fault_skip_kv;              // failure-detection tests: CTA 0 skips this K/V load
 };
 
 
@@ -211,7 +212,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       for (long long x = x_begin; x < x_end && ok;) {
         const Piece pc = piece_at(p, x, x_end);
-        if (piece > 0) ok = mbar_wait(smem_addr(&sm.q_empty), (piece - 1) & 1, abort_flag, WAIT_NS);
+        if (piece > 0) ok = mbar_wait(smem_addr(&sm.q_empty), (piece - 1) & 1, abort_flag, p.wait_ns);
         if (!ok) break;
         const uint32_t bq = smem_addr(&sm.q_full);
         mbar_arrive_expect_tx(bq, 2 * TILE_BYTES);
@@ -223,10 +224,14 @@ __global__ void __launch_bounds__(THREADS, 1)
           for (int hs = 0; hs < pc.kvs && ok; ++hs) {  // one stage per head of the unit
             const int st = nkv % STAGES, h = hs ? pc.ut.h1 : pc.ut.h0;
             if (nkv >= STAGES)
-              ok = mbar_wait(smem_addr(&sm.kv_empty[st]), ((nkv / STAGES) - 1) & 1, abort_flag, WAIT_NS);
+              ok = mbar_wait(smem_addr(&sm.kv_empty[st]), ((nkv / STAGES) - 1) & 1, abort_flag, p.wait_ns);
             if (!ok) break;
             // K and V of the tile land on one barrier: the issuer waits once
             const uint32_t bkv = smem_addr(&sm.kv_full[st]);
+            if (b == 0 && nkv == p.fault_skip_kv) {  // injected fault: nothing lands here
+              ++nkv;
+              continue;
+            }
             mbar_arrive_expect_tx(bkv, 2 * TILE_BYTES);
             if (j < p.nb) {
               tma_load_3d(smem_addr(sm.k[st]), &tmBK, bkv, 0, j * BN, h);
@@ -243,7 +248,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       // Every issued copy must land before the CTA exits; the last load into
       // each stage is the only one that can still be in flight.
       for (int i = nkv - STAGES > 0 ? nkv - STAGES : 0; i < nkv; ++i)
-        mbar_wait(smem_addr(&sm.kv_full[i % STAGES]), (i / STAGES) & 1, never, DRAIN_NS);
+        if (!(b == 0 && i == p.fault_skip_kv))
+          mbar_wait(smem_addr(&sm.kv_full[i % STAGES]), (i / STAGES) & 1, never, DRAIN_NS);
       if (piece > 0) mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, never, DRAIN_NS);
     }
   } else {
@@ -273,16 +279,16 @@ __global__ void __launch_bounds__(THREADS, 1)
           // Q K^T(j) of query tile t goes out once S(j-1) of that tile has
           // been read; the Q tiles are released after the piece's last one,
           // each stage after the Q K^T of both tiles has read its K.
-          ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, WAIT_NS);
+          ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, p.wait_ns);
           for (int jj = 0; jj < n && ok; ++jj) {
             for (int t = 0; t < ntiles && ok; ++t) {
               const int tq = use_of(jj, t), st = tq % STAGES;
               if (t == 0 || pc.kvs == 2) {  // the stage holding this tile's K
-                ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, WAIT_NS);
+                ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, p.wait_ns);
                 if (!ok) break;
               }
               if (jj > 0) {
-                ok = mbar_wait(smem_addr(&sm.s_free[t]), (t ? ph1 : ph0) & 1, abort_flag, WAIT_NS);
+                ok = mbar_wait(smem_addr(&sm.s_free[t]), (t ? ph1 : ph0) & 1, abort_flag, p.wait_ns);
                 if (t) ++ph1; else ++ph0;
                 if (!ok) break;
               }
@@ -300,10 +306,10 @@ __global__ void __launch_bounds__(THREADS, 1)
           mma_commit(smem_addr(&sm.q_empty));
           // the softmax also arrives on s_free for the piece's last tile; the
           // next piece's first Q K^T waits for it
-          if (ok) ok = mbar_wait(smem_addr(&sm.s_free[0]), ph0 & 1, abort_flag, WAIT_NS);
+          if (ok) ok = mbar_wait(smem_addr(&sm.s_free[0]), ph0 & 1, abort_flag, p.wait_ns);
           ++ph0;
           if (ok && ntiles == 2) {
-            ok = mbar_wait(smem_addr(&sm.s_free[1]), ph1 & 1, abort_flag, WAIT_NS);
+            ok = mbar_wait(smem_addr(&sm.s_free[1]), ph1 & 1, abort_flag, p.wait_ns);
             ++ph1;
           }
         } else if (tpv == 0 || pc.ut.has1) {
@@ -314,7 +320,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const uint32_t d_o = tmem + (tpv ? TM_O1 : TM_O0), d_p = tmem + (tpv ? TM_P1 : TM_P0);
           for (int jj = 0; jj < n && ok; ++jj) {
             const int st = use_of(jj, tpv) % STAGES;
-            ok = mbar_wait(b_pready, ph0 & 1, abort_flag, WAIT_NS);
+            ok = mbar_wait(b_pready, ph0 & 1, abort_flag, p.wait_ns);
             ++ph0;
             if (!ok) break;
             tc_fence_after();
@@ -329,7 +335,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               // the other head's stage of this key tile: this issuer's release
               // of it (an arrival only after that use's load has landed)
               const int to = use_of(jj, 1 - tpv), so = to % STAGES;
-              ok = mbar_wait(smem_addr(&sm.kv_full[so]), (to / STAGES) & 1, abort_flag, WAIT_NS);
+              ok = mbar_wait(smem_addr(&sm.kv_full[so]), (to / STAGES) & 1, abort_flag, p.wait_ns);
               if (ok) mbar_arrive(smem_addr(&sm.kv_empty[so]));
             }
           }
@@ -339,7 +345,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           // only after that use's load has landed)
           for (int jj = 0; jj < n && ok; ++jj) {
             const int tq = use_of(jj, 0), st = tq % STAGES;
-            ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, WAIT_NS);
+            ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, p.wait_ns);
             if (ok) mbar_arrive(smem_addr(&sm.kv_empty[st]));
           }
         }
@@ -365,9 +371,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint32_t s_phase = 0, o_phase = 0;  // s_full parity, P V completions consumed
     bool stop = false;
     // Bounded wait for a barrier phase (gives up on the abort word or after
-    // WAIT_NS); a warp stops as a whole if any of its lanes gave up.
+    // p.wait_ns); a warp stops as a whole if any of its lanes gave up.
     auto wait_phase = [&](uint32_t bar, uint32_t parity) -> bool {
-      const bool ok = mbar_wait(bar, parity, abort_flag, WAIT_NS);
+      const bool ok = mbar_wait(bar, parity, abort_flag, p.wait_ns);
       if (__any_sync(0xffffffffu, !ok)) return false;
       tc_fence_after();
       return true;
@@ -578,6 +584,8 @@ Params make_params(const AttnArgs& a) {
   p.status = a.status;
   p.clk_start = a.clk_start;
   p.clk_end = a.clk_end;
+  p.wait_ns = a.wait_ns;
+  p.fault_skip_kv = a.fault_skip_kv;
   return p;
 }
 

@@ -107,6 +107,12 @@ struct AttnArgs {
   // and the latest CTA end (preset to 0)
   unsigned long long* clk_start;
   unsigned long long* clk_end;
+  // limit of every bounded wait in the kernel (ns; 2 s in normal use)
+  unsigned long long wait_ns;
+  // failure-detection tests only: CTA 0's producer does not issue this K/V
+  // load (CTA-local load index), so the bounded waits on its stage run out;
+  // -1 in normal use
+  int fault_skip_kv;
 };
 
 // Work decomposition: a unit is a pair of 128-row query tiles run over all

@@ -184,6 +184,8 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
   a.part_o = sc->part_o;
   a.part_lse = sc->part_lse;
   a.status = st;
+  a.wait_ns = 2000000000ull;  // 2 s
+  a.fault_skip_kv = -1;
   a.grid = (int)G;
   if (launch_attention(a, stream) != cudaSuccess) return REGMEM_ERR_CUDA;
 

@@ -84,6 +84,10 @@ struct regmem {
   int attn_ctas_per_sm = 0;
   int* status_host = nullptr; // mapped pinned word written by kernels
   int* status_dev = nullptr;
+  // bounded waits of the attention kernel, and the one-shot fault of
+  // regmem_debug_set (failure-detection tests)
+  unsigned long long wait_ns = 2000000000ull;
+  int fault_skip_kv = -1;
 
   // staging of the host-buffer entry points (allocated by regmem_set_frame)
   __nv_bfloat16* stQ = nullptr;
@@ -279,6 +283,9 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   a.part_o = h->part_o;
   a.part_lse = h->part_lse;
   a.status = h->status_dev;
+  a.wait_ns = h->wait_ns;
+  a.fault_skip_kv = h->fault_skip_kv;
+  h->fault_skip_kv = -1;  // one launch only
   if (h->kclock && h->time_every > 0 && h->clk_next < kClockSlots) {
     a.clk_start = h->kclock + h->clk_next;
     a.clk_end = h->kclock + kClockSlots + h->clk_next;
@@ -900,6 +907,15 @@ regmem_status regmem_synchronize(regmem_t* h) {
     RM_CUDA(h, cudaGetLastError());
   }
   return check_device_status(h);
+}
+
+regmem_status regmem_debug_set(regmem_t* h, int64_t wait_limit_us, int32_t skip_kv_load) {
+  REGMEM_RANGE;
+  if (!h || wait_limit_us < 1 || wait_limit_us > 60000000 || skip_kv_load < -1)
+    return REGMEM_ERR_ARG;
+  h->wait_ns = (unsigned long long)wait_limit_us * 1000ull;
+  h->fault_skip_kv = skip_kv_load;
+  return REGMEM_OK;
 }
 
 regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention) {

@@ -41,6 +41,7 @@ _SIGNATURES = {
     "regmem_synchronize": (ctypes.c_int, [_P]),
     "regmem_attend_frame_noalloc": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, ctypes.c_int64,
                                                    ctypes.c_int64, _P, _P, _P, _P]),
+    "regmem_debug_set": (ctypes.c_int, [_P, ctypes.c_int64, _I32]),
     "regmem_profile_enable": (ctypes.c_int, [_P, _I32]),
     "regmem_profile_read": (ctypes.c_int, [_P, _P]),
     "regmem_last_error": (ctypes.c_char_p, [_P]),
@@ -237,6 +238,12 @@ def regmem_attend_frame_noalloc(n_special, grid_h, grid_w, heads, Q, K, V, bankK
     return st
 
 
+def regmem_debug_set(h, wait_limit_us=2000000, skip_kv_load=-1):
+    """Failure-detection hook: bounded-wait limit of the attention kernel and
+    a one-shot skipped K/V load in its next launch."""
+    return _check(h, load().regmem_debug_set(h, int(wait_limit_us), int(skip_kv_load)))
+
+
 def regmem_profile_enable(h, time_attention=1):
     return _check(h, load().regmem_profile_enable(h, int(time_attention)))
 
@@ -322,6 +329,9 @@ class RegMem:
 
     def synchronize(self):
         return regmem_synchronize(self.h)
+
+    def debug_set(self, wait_limit_us=2000000, skip_kv_load=-1):
+        return regmem_debug_set(self.h, wait_limit_us, skip_kv_load)
 
     def profile_enable(self, time_attention=1):
         return regmem_profile_enable(self.h, time_attention)
