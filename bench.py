@@ -74,7 +74,7 @@ CONFIGS = {
 # {(config, attended rows L): bytes}.  The line reports the capture whose L
 # lies within 2 % of the timed launches' mean L, else null; the table is
 # emptied whenever the attention kernel changes until it is captured again.
-ATTN_TRAFFIC_CAPTURES = {}
+ATTN_TRAFFIC_CAPTURES = {("long", 16734): 73.64e6, ("long", 30720): 501.2e6}
 
 
 def traffic_for(cfg_name, mean_L):
@@ -651,7 +651,7 @@ def gpu_arm(args, cfg, cfg_name):
             "traffic": traffic[0],
             "traffic_note": traffic[1],
             "launches": prof.attention_clocked or prof.attention_timed,
-            "launches_total": prof.launches_attention,
+            "launches_total": prof.launches_attention - prof.launches_frame_attention,
             "ctas": prof.attention_ctas,
             "ctas_per_sm": prof.attention_ctas_per_sm,
             "mean_launch_ms": round(roof_ms_mean, 5),
@@ -671,13 +671,27 @@ def gpu_arm(args, cfg, cfg_name):
                 "merge_mean_ms": round(merge_ms_mean, 5),
             },
             # attention kernel plus the merge of split units behind it
-            "share_of_step": (round((roof_ms_mean + merge_ms_mean) * prof.launches_attention / ms_local, 4)
+            "share_of_step": (round((roof_ms_mean * (prof.launches_attention - prof.launches_frame_attention)
+                                     + prof.frame_attention_clock_ms
+                                     + merge_ms_mean * prof.launches_attention) / ms_local, 4)
                               if ms_local else None),
         },
         "gpu_launches": launches,
         "clocks": clk,
         "e2e": e2e,
     }
+    if cfg["fa"] and prof.frame_attention_clocked:
+        # the non-causal frame-attention layers (Sec. 3.1) run the same kernel
+        # with no memory: their own launch clock and algorithmic FLOPs
+        fa_ms = prof.frame_attention_clock_ms / prof.frame_attention_clocked
+        fa_flops = prof.frame_attention_clock_flops / prof.frame_attention_clocked
+        fa_tf = fa_flops / (fa_ms / 1e3) / 1e12 if fa_ms else 0.0
+        line["roofline_frame_attention"] = {
+            "kernel": "attn_fwd_kernel on the frame's own N keys (regmem_frame_attention)",
+            "bound": "tensor", "achieved": round(fa_tf, 2), "peak": peak, "unit": "TFLOP/s",
+            "frac": round(fa_tf / peak, 4), "launches": prof.frame_attention_clocked,
+            "mean_launch_ms": round(fa_ms, 5), "algorithmic_flops_per_launch": fa_flops,
+        }
     if cfg.get("variant"):
         share = line["roofline"]["share_of_step"] or 0.0
         line["memory"] = {

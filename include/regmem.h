@@ -330,9 +330,15 @@ typedef struct regmem_profile {
   int32_t attention_ctas_per_sm; /* resident attention CTAs per SM (occupancy) */
   double merge_ms;            /* summed event time of the merges of split units
                                  behind those launches                          */
-  int64_t attention_clocked;  /* attention launches measured by the launch clock */
+  int64_t attention_clocked;  /* regulated attention launches (attend calls)
+                                 measured by the launch clock                   */
   double attention_clock_ms;  /* their summed durations (global timer)          */
   double attention_clock_flops; /* algorithmic FLOPs of those launches          */
+  int64_t launches_frame_attention; /* of launches_attention: regmem_frame_attention */
+  int64_t frame_attention_clocked;  /* frame-attention launches measured by the
+                                       launch clock                              */
+  double frame_attention_clock_ms;  /* their summed durations                   */
+  double frame_attention_clock_flops; /* their algorithmic FLOPs, 4 N^2 64 H each */
 } regmem_profile;
 
 /* Resets the counters; time_attention = n >= 1 also brackets every n-th

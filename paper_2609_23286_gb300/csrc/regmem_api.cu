@@ -79,6 +79,7 @@ struct regmem {
   // words, one pair per launch since regmem_profile_enable
   unsigned long long* kclock = nullptr;
   long long clk_next = 0;
+  std::vector<unsigned char> clk_frame;  // per clocked launch: 1 = frame attention
   uint64_t* adm_lists = nullptr;  // per-(head, key tile) candidate lists, [H][nkt][32]
   int attn_grid = 0;
   int attn_ctas_per_sm = 0;
@@ -254,7 +255,7 @@ regmem_status join_side(regmem_t* h) {
 }
 
 regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K, const void* V,
-                            void* out, int M) {
+                            void* out, int M, bool frame_attention = false) {
   // the layer's previous saliency and admission (side stream) read its LSE
   // rows and append to its bank: they finish before this attention starts.
   // One wait covers all side work so far, so in a stream of frames only the
@@ -289,6 +290,7 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   if (h->kclock && h->time_every > 0 && h->clk_next < kClockSlots) {
     a.clk_start = h->kclock + h->clk_next;
     a.clk_end = h->kclock + kClockSlots + h->clk_next;
+    h->clk_frame[h->clk_next] = frame_attention ? 1 : 0;
     ++h->clk_next;
   }
   const AttnPlan pl = attn_plan(h->N, h->heads, M);
@@ -317,7 +319,12 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   const double L = (double)M + h->N;
   h->prof.launches_attention += 1;
   if (a.grid > 1) h->prof.launches_combine += 1;
-  if (a.clk_start) h->prof.attention_clock_flops += 4.0 * h->N * L * kHeadDim * h->heads;
+  if (frame_attention) h->prof.launches_frame_attention += 1;
+  if (a.clk_start) {
+    const double flops = 4.0 * h->N * L * kHeadDim * h->heads;
+    if (frame_attention) h->prof.frame_attention_clock_flops += flops;
+    else h->prof.attention_clock_flops += flops;
+  }
   if (timed) {
     h->prof.attention_timed += 1;
     h->prof.attention_flops += 4.0 * h->N * L * kHeadDim * h->heads;
@@ -811,7 +818,7 @@ regmem_status regmem_frame_attention(regmem_t* h, const void* Q, const void* K, 
   if (!Q || !K || !V || !out) return fail(h, REGMEM_ERR_ARG, "null tensor pointer");
   if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(out))
     return fail(h, REGMEM_ERR_ARG, "tensor pointers must be 16-byte aligned");
-  return run_attention(h, 0, Q, K, V, out, 0);
+  return run_attention(h, 0, Q, K, V, out, 0, true);
 }
 
 regmem_status regmem_reset(regmem_t* h) {
@@ -933,6 +940,7 @@ regmem_status regmem_profile_enable(regmem_t* h, int32_t time_attention) {
   if (h->frame_set && h->time_every > 0) {  // preset the slots, stream-ordered before the launches
     const size_t bytes = 2 * kClockSlots * sizeof(unsigned long long);
     if (!h->kclock) RM_CUDA(h, cudaMalloc(&h->kclock, bytes));
+    h->clk_frame.assign(kClockSlots, 0);
     RM_CUDA(h, cudaMemsetAsync(h->kclock, 0xFF, bytes / 2, h->stream));
     RM_CUDA(h, cudaMemsetAsync(h->kclock + kClockSlots, 0, bytes / 2, h->stream));
   }
@@ -956,11 +964,17 @@ regmem_status regmem_profile_read(regmem_t* h, regmem_profile* out) {
                             cudaMemcpyDeviceToHost));
       RM_CUDA(h, cudaMemcpy(t1.data(), h->kclock + kClockSlots, n * sizeof(unsigned long long),
                             cudaMemcpyDeviceToHost));
-      double ns = 0.0;
-      for (size_t i = 0; i < n; ++i)
-        if (t1[i] > t0[i]) ns += (double)(t1[i] - t0[i]);
-      h->prof.attention_clocked = h->clk_next;
-      h->prof.attention_clock_ms = ns * 1e-6;
+      double ns[2] = {0.0, 0.0};
+      long long cnt[2] = {0, 0};
+      for (size_t i = 0; i < n; ++i) {
+        const int f = h->clk_frame[i];
+        ++cnt[f];
+        if (t1[i] > t0[i]) ns[f] += (double)(t1[i] - t0[i]);
+      }
+      h->prof.attention_clocked = cnt[0];
+      h->prof.attention_clock_ms = ns[0] * 1e-6;
+      h->prof.frame_attention_clocked = cnt[1];
+      h->prof.frame_attention_clock_ms = ns[1] * 1e-6;
     }
   }
   *out = h->prof;

@@ -67,7 +67,11 @@ class Profile(ctypes.Structure):
                 ("attention_bytes", ctypes.c_double), ("attention_ctas", ctypes.c_int32),
                 ("attention_ctas_per_sm", ctypes.c_int32), ("merge_ms", ctypes.c_double),
                 ("attention_clocked", ctypes.c_int64), ("attention_clock_ms", ctypes.c_double),
-                ("attention_clock_flops", ctypes.c_double)]
+                ("attention_clock_flops", ctypes.c_double),
+                ("launches_frame_attention", ctypes.c_int64),
+                ("frame_attention_clocked", ctypes.c_int64),
+                ("frame_attention_clock_ms", ctypes.c_double),
+                ("frame_attention_clock_flops", ctypes.c_double)]
 
     def as_dict(self):
         return {f: getattr(self, f) for f, _ in self._fields_}
