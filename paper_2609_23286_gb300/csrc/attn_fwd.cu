@@ -115,15 +115,16 @@ constexpr size_t SMEM_BYTES = (sizeof(Smem) + 127) & ~size_t(127);
 static_assert(SMEM_BYTES <= 232448, "more dynamic shared memory than a CTA can have (227 KB)");
 
 struct Params {
-  SplitBounds bnd;  // this launch's split: CTA b takes tiles [bnd.x[b], bnd.x[b + 1])
+  SplitBounds bnd;  // this launch's split: CTA b takes tiles [bnd.x[p][b], bnd.x[p][b + 1]) of phase p
   int N, H, M;
   int nb, nkv, nqt;
   long long total;
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  __nv_bfloat16* part_o;  // [grid][2][256][64]: partials of each CTA's first / last piece
-  float* part_lse;  // [grid][2][256]
+  __nv_bfloat16* part_o;  // [grid][bnd.slots][256][64]: partials of each CTA's first / last
+                          // piece of each phase
+  float* part_lse;  // [grid][bnd.slots][256]
   int* status;
   unsigned long long* clk_start;  // launch clock (AttnArgs) or nullptr
   unsigned long long* clk_end;
@@ -167,7 +168,6 @@ __global__ void __launch_bounds__(THREADS, 1)
   volatile int* never = &sm.never;
 
   const int G = gridDim.x, b = blockIdx.x;
-  const long long x_begin = p.bnd.x[b], x_end = p.bnd.x[b + 1];
 
   if (tid == 0) {
     sm.abort_flag = 0;
@@ -210,40 +210,43 @@ __global__ void __launch_bounds__(THREADS, 1)
       prefetch_tmap(&tmBV);
       int nkv = 0, piece = 0;  // K/V tile pairs, Q pairs issued
       bool ok = true;
-      for (long long x = x_begin; x < x_end && ok;) {
-        const Piece pc = piece_at(p, x, x_end);
-        if (piece > 0) ok = mbar_wait(smem_addr(&sm.q_empty), (piece - 1) & 1, abort_flag, p.wait_ns);
-        if (!ok) break;
-        const uint32_t bq = smem_addr(&sm.q_full);
-        mbar_arrive_expect_tx(bq, 2 * TILE_BYTES);
-        // (a unit without a second tile loads rows past the frame: zero fill)
-        tma_load_3d(smem_addr(sm.q[0]), &tmQ, bq, 0, pc.ut.h0, pc.ut.qt0 * BM);
-        tma_load_3d(smem_addr(sm.q[1]), &tmQ, bq, 0, pc.ut.h1, pc.ut.qt1 * BM);
-        ++piece;
-        for (int j = pc.j0; j < pc.j1 && ok; ++j) {
-          for (int hs = 0; hs < pc.kvs && ok; ++hs) {  // one stage per head of the unit
-            const int st = nkv % STAGES, h = hs ? pc.ut.h1 : pc.ut.h0;
-            if (nkv >= STAGES)
-              ok = mbar_wait(smem_addr(&sm.kv_empty[st]), ((nkv / STAGES) - 1) & 1, abort_flag, p.wait_ns);
-            if (!ok) break;
-            // K and V of the tile land on one barrier: the issuer waits once
-            const uint32_t bkv = smem_addr(&sm.kv_full[st]);
-            if (b == 0 && nkv == p.fault_skip_kv) {  // injected fault: nothing lands here
+      for (int ph = 0; ph < p.bnd.P && ok; ++ph) {
+        const long long x_begin = p.bnd.x[ph][b], x_end = p.bnd.x[ph][b + 1];
+        for (long long x = x_begin; x < x_end && ok;) {
+          const Piece pc = piece_at(p, x, x_end);
+          if (piece > 0) ok = mbar_wait(smem_addr(&sm.q_empty), (piece - 1) & 1, abort_flag, p.wait_ns);
+          if (!ok) break;
+          const uint32_t bq = smem_addr(&sm.q_full);
+          mbar_arrive_expect_tx(bq, 2 * TILE_BYTES);
+          // (a unit without a second tile loads rows past the frame: zero fill)
+          tma_load_3d(smem_addr(sm.q[0]), &tmQ, bq, 0, pc.ut.h0, pc.ut.qt0 * BM);
+          tma_load_3d(smem_addr(sm.q[1]), &tmQ, bq, 0, pc.ut.h1, pc.ut.qt1 * BM);
+          ++piece;
+          for (int j = pc.j0; j < pc.j1 && ok; ++j) {
+            for (int hs = 0; hs < pc.kvs && ok; ++hs) {  // one stage per head of the unit
+              const int st = nkv % STAGES, h = hs ? pc.ut.h1 : pc.ut.h0;
+              if (nkv >= STAGES)
+                ok = mbar_wait(smem_addr(&sm.kv_empty[st]), ((nkv / STAGES) - 1) & 1, abort_flag, p.wait_ns);
+              if (!ok) break;
+              // K and V of the tile land on one barrier: the issuer waits once
+              const uint32_t bkv = smem_addr(&sm.kv_full[st]);
+              if (b == 0 && nkv == p.fault_skip_kv) {  // injected fault: nothing lands here
+                ++nkv;
+                continue;
+              }
+              mbar_arrive_expect_tx(bkv, 2 * TILE_BYTES);
+              if (j < p.nb) {
+                tma_load_3d(smem_addr(sm.k[st]), &tmBK, bkv, 0, j * BN, h);
+                tma_load_3d(smem_addr(sm.v[st]), &tmBV, bkv, 0, j * BN, h);
+              } else {
+                tma_load_3d(smem_addr(sm.k[st]), &tmK, bkv, 0, h, (j - p.nb) * BN);
+                tma_load_3d(smem_addr(sm.v[st]), &tmV, bkv, 0, h, (j - p.nb) * BN);
+              }
               ++nkv;
-              continue;
             }
-            mbar_arrive_expect_tx(bkv, 2 * TILE_BYTES);
-            if (j < p.nb) {
-              tma_load_3d(smem_addr(sm.k[st]), &tmBK, bkv, 0, j * BN, h);
-              tma_load_3d(smem_addr(sm.v[st]), &tmBV, bkv, 0, j * BN, h);
-            } else {
-              tma_load_3d(smem_addr(sm.k[st]), &tmK, bkv, 0, h, (j - p.nb) * BN);
-              tma_load_3d(smem_addr(sm.v[st]), &tmV, bkv, 0, h, (j - p.nb) * BN);
-            }
-            ++nkv;
           }
+          x += pc.j1 - pc.j0;
         }
-        x += pc.j1 - pc.j0;
       }
       // Every issued copy must land before the CTA exits; the last load into
       // each stage is the only one that can still be in flight.
@@ -264,89 +267,92 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t ph0 = 0, ph1 = 0;  // s_free (QK) or p_ready (PV) phases consumed, per query tile
       int it = 0, piece = 0;
       bool ok = true;
-      for (long long x = x_begin; x < x_end && ok;) {
-        const Piece pc = piece_at(p, x, x_end);
-        const int n = pc.j1 - pc.j0;
-        x += n;
-        ++piece;
-        const int ntiles = pc.ut.has1 ? 2 : 1;  // query tiles of this unit
-        // CTA-local stage use of key tile jj for query tile t: one stage per
-        // key tile, or two (one per head) when the tiles belong to two heads
-        const int t0 = it;
-        it += n * pc.kvs;
-        auto use_of = [&](int jj, int t) { return t0 + jj * pc.kvs + (pc.kvs == 2 ? t : 0); };
-        if (qk_role) {
-          // Q K^T(j) of query tile t goes out once S(j-1) of that tile has
-          // been read; the Q tiles are released after the piece's last one,
-          // each stage after the Q K^T of both tiles has read its K.
-          ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, p.wait_ns);
-          for (int jj = 0; jj < n && ok; ++jj) {
-            for (int t = 0; t < ntiles && ok; ++t) {
-              const int tq = use_of(jj, t), st = tq % STAGES;
-              if (t == 0 || pc.kvs == 2) {  // the stage holding this tile's K
-                ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, p.wait_ns);
-                if (!ok) break;
+      for (int ph = 0; ph < p.bnd.P && ok; ++ph) {
+        const long long x_begin = p.bnd.x[ph][b], x_end = p.bnd.x[ph][b + 1];
+        for (long long x = x_begin; x < x_end && ok;) {
+          const Piece pc = piece_at(p, x, x_end);
+          const int n = pc.j1 - pc.j0;
+          x += n;
+          ++piece;
+          const int ntiles = pc.ut.has1 ? 2 : 1;  // query tiles of this unit
+          // CTA-local stage use of key tile jj for query tile t: one stage per
+          // key tile, or two (one per head) when the tiles belong to two heads
+          const int t0 = it;
+          it += n * pc.kvs;
+          auto use_of = [&](int jj, int t) { return t0 + jj * pc.kvs + (pc.kvs == 2 ? t : 0); };
+          if (qk_role) {
+            // Q K^T(j) of query tile t goes out once S(j-1) of that tile has
+            // been read; the Q tiles are released after the piece's last one,
+            // each stage after the Q K^T of both tiles has read its K.
+            ok = mbar_wait(smem_addr(&sm.q_full), (piece - 1) & 1, abort_flag, p.wait_ns);
+            for (int jj = 0; jj < n && ok; ++jj) {
+              for (int t = 0; t < ntiles && ok; ++t) {
+                const int tq = use_of(jj, t), st = tq % STAGES;
+                if (t == 0 || pc.kvs == 2) {  // the stage holding this tile's K
+                  ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, p.wait_ns);
+                  if (!ok) break;
+                }
+                if (jj > 0) {
+                  ok = mbar_wait(smem_addr(&sm.s_free[t]), (t ? ph1 : ph0) & 1, abort_flag, p.wait_ns);
+                  if (t) ++ph1; else ++ph0;
+                  if (!ok) break;
+                }
+                tc_fence_after();
+                const uint32_t sq = smem_addr(sm.q[t]), d_s = tmem + (t ? TM_S1 : TM_S0);
+                const uint32_t kaddr = smem_addr(sm.k[st]);
+  #pragma unroll
+                for (int kk = 0; kk < HD / 16; ++kk)
+                  mma_ss(d_s, sdesc_sw128(sq + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
+                mma_commit(smem_addr(&sm.s_full[t]));
+                // the stage's K is read by the last Q K^T that uses it
+                if (t == ntiles - 1 || pc.kvs == 2) mma_commit(smem_addr(&sm.kv_empty[st]));
               }
-              if (jj > 0) {
-                ok = mbar_wait(smem_addr(&sm.s_free[t]), (t ? ph1 : ph0) & 1, abort_flag, p.wait_ns);
-                if (t) ++ph1; else ++ph0;
-                if (!ok) break;
-              }
-              tc_fence_after();
-              const uint32_t sq = smem_addr(sm.q[t]), d_s = tmem + (t ? TM_S1 : TM_S0);
-              const uint32_t kaddr = smem_addr(sm.k[st]);
-#pragma unroll
-              for (int kk = 0; kk < HD / 16; ++kk)
-                mma_ss(d_s, sdesc_sw128(sq + kk * 32), sdesc_sw128(kaddr + kk * 32), IDESC_QK, kk > 0);
-              mma_commit(smem_addr(&sm.s_full[t]));
-              // the stage's K is read by the last Q K^T that uses it
-              if (t == ntiles - 1 || pc.kvs == 2) mma_commit(smem_addr(&sm.kv_empty[st]));
             }
-          }
-          mma_commit(smem_addr(&sm.q_empty));
-          // the softmax also arrives on s_free for the piece's last tile; the
-          // next piece's first Q K^T waits for it
-          if (ok) ok = mbar_wait(smem_addr(&sm.s_free[0]), ph0 & 1, abort_flag, p.wait_ns);
-          ++ph0;
-          if (ok && ntiles == 2) {
-            ok = mbar_wait(smem_addr(&sm.s_free[1]), ph1 & 1, abort_flag, p.wait_ns);
-            ++ph1;
-          }
-        } else if (tpv == 0 || pc.ut.has1) {
-          // P V(j) of the query tile goes out once P(j) is stored; its
-          // completion releases P (o_done, waited by the softmax) and the
-          // stage (the last read of its V).  The issuer does not wait for it.
-          const uint32_t b_pready = smem_addr(&sm.p_ready[tpv]), b_odone = smem_addr(&sm.o_done[tpv]);
-          const uint32_t d_o = tmem + (tpv ? TM_O1 : TM_O0), d_p = tmem + (tpv ? TM_P1 : TM_P0);
-          for (int jj = 0; jj < n && ok; ++jj) {
-            const int st = use_of(jj, tpv) % STAGES;
-            ok = mbar_wait(b_pready, ph0 & 1, abort_flag, p.wait_ns);
+            mma_commit(smem_addr(&sm.q_empty));
+            // the softmax also arrives on s_free for the piece's last tile; the
+            // next piece's first Q K^T waits for it
+            if (ok) ok = mbar_wait(smem_addr(&sm.s_free[0]), ph0 & 1, abort_flag, p.wait_ns);
             ++ph0;
-            if (!ok) break;
-            tc_fence_after();
-            const uint32_t vaddr = smem_addr(sm.v[st]);
-#pragma unroll
-            for (int kk = 0; kk < BN / 16; ++kk)  // 16 keys = 8 packed columns of P
-              mma_ts(d_o, d_p + kk * 8, sdesc_sw128(vaddr + kk * 2048), IDESC_PV,
-                     (jj == 0 && kk == 0) ? 0u : 1u);
-            mma_commit(b_odone);
-            mma_commit(smem_addr(&sm.kv_empty[st]));
-            if (ok && pc.kvs == 2) {
-              // the other head's stage of this key tile: this issuer's release
-              // of it (an arrival only after that use's load has landed)
-              const int to = use_of(jj, 1 - tpv), so = to % STAGES;
-              ok = mbar_wait(smem_addr(&sm.kv_full[so]), (to / STAGES) & 1, abort_flag, p.wait_ns);
-              if (ok) mbar_arrive(smem_addr(&sm.kv_empty[so]));
+            if (ok && ntiles == 2) {
+              ok = mbar_wait(smem_addr(&sm.s_free[1]), ph1 & 1, abort_flag, p.wait_ns);
+              ++ph1;
             }
-          }
-        } else {
-          // tile 1 of a unit without one: nothing to compute, but the stage
-          // releases keep their order (an arrival for a stage's next use
-          // only after that use's load has landed)
-          for (int jj = 0; jj < n && ok; ++jj) {
-            const int tq = use_of(jj, 0), st = tq % STAGES;
-            ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, p.wait_ns);
-            if (ok) mbar_arrive(smem_addr(&sm.kv_empty[st]));
+          } else if (tpv == 0 || pc.ut.has1) {
+            // P V(j) of the query tile goes out once P(j) is stored; its
+            // completion releases P (o_done, waited by the softmax) and the
+            // stage (the last read of its V).  The issuer does not wait for it.
+            const uint32_t b_pready = smem_addr(&sm.p_ready[tpv]), b_odone = smem_addr(&sm.o_done[tpv]);
+            const uint32_t d_o = tmem + (tpv ? TM_O1 : TM_O0), d_p = tmem + (tpv ? TM_P1 : TM_P0);
+            for (int jj = 0; jj < n && ok; ++jj) {
+              const int st = use_of(jj, tpv) % STAGES;
+              ok = mbar_wait(b_pready, ph0 & 1, abort_flag, p.wait_ns);
+              ++ph0;
+              if (!ok) break;
+              tc_fence_after();
+              const uint32_t vaddr = smem_addr(sm.v[st]);
+  #pragma unroll
+              for (int kk = 0; kk < BN / 16; ++kk)  // 16 keys = 8 packed columns of P
+                mma_ts(d_o, d_p + kk * 8, sdesc_sw128(vaddr + kk * 2048), IDESC_PV,
+                       (jj == 0 && kk == 0) ? 0u : 1u);
+              mma_commit(b_odone);
+              mma_commit(smem_addr(&sm.kv_empty[st]));
+              if (ok && pc.kvs == 2) {
+                // the other head's stage of this key tile: this issuer's release
+                // of it (an arrival only after that use's load has landed)
+                const int to = use_of(jj, 1 - tpv), so = to % STAGES;
+                ok = mbar_wait(smem_addr(&sm.kv_full[so]), (to / STAGES) & 1, abort_flag, p.wait_ns);
+                if (ok) mbar_arrive(smem_addr(&sm.kv_empty[so]));
+              }
+            }
+          } else {
+            // tile 1 of a unit without one: nothing to compute, but the stage
+            // releases keep their order (an arrival for a stage's next use
+            // only after that use's load has landed)
+            for (int jj = 0; jj < n && ok; ++jj) {
+              const int tq = use_of(jj, 0), st = tq % STAGES;
+              ok = mbar_wait(smem_addr(&sm.kv_full[st]), (tq / STAGES) & 1, abort_flag, p.wait_ns);
+              if (ok) mbar_arrive(smem_addr(&sm.kv_empty[st]));
+            }
           }
         }
       }
@@ -382,117 +388,140 @@ __global__ void __launch_bounds__(THREADS, 1)
     // is in registers, waits for P V(j-1) (P is single-buffered) before
     // storing P(j), and arrives on p_ready once P(j) is stored.  Every thread
     // arrives (cheaper than a warp-elected arrival after a warp barrier).
-    for (long long x = x_begin; x < x_end && !stop;) {
-      const Piece pc = piece_at(p, x, x_end);
-      const int n = pc.j1 - pc.j0;
-      x += n;
-      if (t == 1 && !pc.ut.has1) continue;  // no rows in this unit's second tile
-      const int th = t ? pc.ut.h1 : pc.ut.h0, tqt = t ? pc.ut.qt1 : pc.ut.qt0;  // this tile's head, index
-      float m_used = -INFINITY;  // running max of the logits, scaled to log2 units
-      float l = 0.f;             // running row sum of exp2(z*c - m_used)
-      for (int jj = 0; jj < n; ++jj) {
-        const int j = pc.j0 + jj;
-        if (!wait_phase(b_sfull, s_phase)) {  // S(j) in TMEM
-          stop = true;
-          break;
-        }
-        s_phase ^= 1;
-        uint32_t sr[128];
-        tmem_ld128(tm_s, sr);
-        tc_fence_before();
-        mbar_arrive(b_sfree);  // S may be overwritten by the next Q K^T
-        const int valid = tile_valid(p, j);
-        if (valid < BN) {
-#pragma unroll
-          for (int i = 0; i < 128; ++i)
-            if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
-        }
-        // row max: four independent chains of three-input max
-        float mx4[4];
-#pragma unroll
-        for (int a = 0; a < 4; ++a) mx4[a] = __uint_as_float(sr[a]);
-#pragma unroll
-        for (int i = 4; i < 124; i += 8) {
-#pragma unroll
-          for (int a = 0; a < 4; ++a)
-            mx4[a] = fmax3(mx4[a], __uint_as_float(sr[i + 2 * a]), __uint_as_float(sr[i + 2 * a + 1]));
-        }
-        mx4[0] = fmax3(mx4[0], __uint_as_float(sr[124]), __uint_as_float(sr[125]));
-        mx4[1] = fmax3(mx4[1], __uint_as_float(sr[126]), __uint_as_float(sr[127]));
-        const float mx = fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3]));
-        const float mnew = mx * c;
-        float alpha = 1.f;
-        const bool need = mnew > m_used + RESCALE_LOG2;
-        if (need) {
-          alpha = ex2(m_used - mnew);  // 0 on the first tile (m_used = -inf)
-          l *= alpha;
-          m_used = mnew;
-        }
-        // p = exp2(z * c - m_used): packed FMA for the argument, MUFU exp2,
-        // packed ADD for the row sum, bf16x2 pack.  P is computed in registers
-        // before its TMEM columns are known to be free.
-        const uint64_t cc = f2_pack(c, c), nn = f2_pack(-m_used, -m_used);
-        uint64_t acc2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
-        uint32_t pk[2][32];
-#pragma unroll
-        for (int hf = 0; hf < 2; ++hf) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int e = hf * 64 + 2 * i;
-            float a0, a1;
-            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), cc, nn), a0, a1);
-            const float p0 = ex2(a0), p1 = ex2(a1);
-            acc2[i & 1] = f2_add(acc2[i & 1], f2_pack(p0, p1));
-            pk[hf][i] = pack_bf16x2(p0, p1);
-          }
-        }
-        if (jj > 0) {
-          // P V(j-1) has read P and added into O (at most one P V of this
-          // tile is outstanding here, so the parity is unambiguous)
-          if (!wait_phase(b_odone, (o_phase++) & 1)) {
+    for (int ph = 0; ph < p.bnd.P && !stop; ++ph) {
+      const long long x_begin = p.bnd.x[ph][b], x_end = p.bnd.x[ph][b + 1];
+      for (long long x = x_begin; x < x_end && !stop;) {
+        const Piece pc = piece_at(p, x, x_end);
+        const int n = pc.j1 - pc.j0;
+        x += n;
+        if (t == 1 && !pc.ut.has1) continue;  // no rows in this unit's second tile
+        const int th = t ? pc.ut.h1 : pc.ut.h0, tqt = t ? pc.ut.qt1 : pc.ut.qt0;  // this tile's head, index
+        float m_used = -INFINITY;  // running max of the logits, scaled to log2 units
+        float l = 0.f;             // running row sum of exp2(z*c - m_used)
+        for (int jj = 0; jj < n; ++jj) {
+          const int j = pc.j0 + jj;
+          if (!wait_phase(b_sfull, s_phase)) {  // S(j) in TMEM
             stop = true;
             break;
           }
-          if (__any_sync(0xffffffffu, need)) {
-            // rare (the max grew by > 2^8): rescale O before P V(j) adds to it
-#pragma unroll 1
-            for (int hc = 0; hc < 2; ++hc) {  // 32 columns at a time
-              uint32_t orr[32];
-              tmem_ld32(tm_o + 32 * hc, orr);
-#pragma unroll
-              for (int i = 0; i < 32; ++i) orr[i] = __float_as_uint(__uint_as_float(orr[i]) * alpha);
-              tmem_st32(tm_o + 32 * hc, orr);
+          s_phase ^= 1;
+          uint32_t sr[128];
+          tmem_ld128(tm_s, sr);
+          tc_fence_before();
+          mbar_arrive(b_sfree);  // S may be overwritten by the next Q K^T
+          const int valid = tile_valid(p, j);
+          if (valid < BN) {
+  #pragma unroll
+            for (int i = 0; i < 128; ++i)
+              if (i >= valid) sr[i] = __float_as_uint(-INFINITY);
+          }
+          // row max: four independent chains of three-input max
+          float mx4[4];
+  #pragma unroll
+          for (int a = 0; a < 4; ++a) mx4[a] = __uint_as_float(sr[a]);
+  #pragma unroll
+          for (int i = 4; i < 124; i += 8) {
+  #pragma unroll
+            for (int a = 0; a < 4; ++a)
+              mx4[a] = fmax3(mx4[a], __uint_as_float(sr[i + 2 * a]), __uint_as_float(sr[i + 2 * a + 1]));
+          }
+          mx4[0] = fmax3(mx4[0], __uint_as_float(sr[124]), __uint_as_float(sr[125]));
+          mx4[1] = fmax3(mx4[1], __uint_as_float(sr[126]), __uint_as_float(sr[127]));
+          const float mx = fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3]));
+          const float mnew = mx * c;
+          float alpha = 1.f;
+          const bool need = mnew > m_used + RESCALE_LOG2;
+          if (need) {
+            alpha = ex2(m_used - mnew);  // 0 on the first tile (m_used = -inf)
+            l *= alpha;
+            m_used = mnew;
+          }
+          // p = exp2(z * c - m_used): packed FMA for the argument, MUFU exp2,
+          // packed ADD for the row sum, bf16x2 pack.  P is computed in registers
+          // before its TMEM columns are known to be free.
+          const uint64_t cc = f2_pack(c, c), nn = f2_pack(-m_used, -m_used);
+          uint64_t acc2[2] = {f2_pack(0.f, 0.f), f2_pack(0.f, 0.f)};
+          uint32_t pk[2][32];
+  #pragma unroll
+          for (int hf = 0; hf < 2; ++hf) {
+  #pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int e = hf * 64 + 2 * i;
+              float a0, a1;
+              f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), cc, nn), a0, a1);
+              const float p0 = ex2(a0), p1 = ex2(a1);
+              acc2[i & 1] = f2_add(acc2[i & 1], f2_pack(p0, p1));
+              pk[hf][i] = pack_bf16x2(p0, p1);
             }
           }
+          if (jj > 0) {
+            // P V(j-1) has read P and added into O (at most one P V of this
+            // tile is outstanding here, so the parity is unambiguous)
+            if (!wait_phase(b_odone, (o_phase++) & 1)) {
+              stop = true;
+              break;
+            }
+            if (__any_sync(0xffffffffu, need)) {
+              // rare (the max grew by > 2^8): rescale O before P V(j) adds to it
+  #pragma unroll 1
+              for (int hc = 0; hc < 2; ++hc) {  // 32 columns at a time
+                uint32_t orr[32];
+                tmem_ld32(tm_o + 32 * hc, orr);
+  #pragma unroll
+                for (int i = 0; i < 32; ++i) orr[i] = __float_as_uint(__uint_as_float(orr[i]) * alpha);
+                tmem_st32(tm_o + 32 * hc, orr);
+              }
+            }
+          }
+          tmem_st32_async(tm_p, pk[0]);
+          tmem_st32_async(tm_p + 32, pk[1]);
+          tmem_wait_st();
+          tc_fence_before();
+          mbar_arrive(b_pready);
+          {
+            float s0, s1, s2, s3;
+            f2_unpack(acc2[0], s0, s1);
+            f2_unpack(acc2[1], s2, s3);
+            l += (s0 + s1) + (s2 + s3);
+          }
         }
-        tmem_st32_async(tm_p, pk[0]);
-        tmem_st32_async(tm_p + 32, pk[1]);
-        tmem_wait_st();
+        if (stop) break;
+        // -------------------------------------------------------------- epilogue
+        if (!wait_phase(b_odone, (o_phase++) & 1)) {  // the last tile's P V
+          stop = true;
+          break;
+        }
+        uint32_t orr[64];
+        tmem_ld64(tm_o, orr);
         tc_fence_before();
-        mbar_arrive(b_pready);
-        {
-          float s0, s1, s2, s3;
-          f2_unpack(acc2[0], s0, s1);
-          f2_unpack(acc2[1], s2, s3);
-          l += (s0 + s1) + (s2 + s3);
-        }
-      }
-      if (stop) break;
-      // -------------------------------------------------------------- epilogue
-      if (!wait_phase(b_odone, (o_phase++) & 1)) {  // the last tile's P V
-        stop = true;
-        break;
-      }
-      uint32_t orr[64];
-      tmem_ld64(tm_o, orr);
-      tc_fence_before();
-      const float inv_l = 1.f / l;
-      const float lse_val = (m_used + __log2f(l)) * 0.69314718055994531f;
-      const int q = tqt * BM + row;
-      if (pc.j0 == 0 && pc.j1 == p.nkv) {
-        if (q < p.N) {
-          uint4* dst = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + th) * HD);
-#pragma unroll
+        const float inv_l = 1.f / l;
+        const float lse_val = (m_used + __log2f(l)) * 0.69314718055994531f;
+        const int q = tqt * BM + row;
+        if (pc.j0 == 0 && pc.j1 == p.nkv) {
+          if (q < p.N) {
+            uint4* dst = reinterpret_cast<uint4*>(p.out + ((size_t)q * p.H + th) * HD);
+  #pragma unroll
+            for (int c8 = 0; c8 < 8; ++c8) {
+              uint4 w;
+              w.x = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 0]) * inv_l, __uint_as_float(orr[c8 * 8 + 1]) * inv_l);
+              w.y = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 2]) * inv_l, __uint_as_float(orr[c8 * 8 + 3]) * inv_l);
+              w.z = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 4]) * inv_l, __uint_as_float(orr[c8 * 8 + 5]) * inv_l);
+              w.w = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 6]) * inv_l, __uint_as_float(orr[c8 * 8 + 7]) * inv_l);
+              dst[c8] = w;
+            }
+            p.lse[(size_t)th * p.N + q] = lse_val;
+          }
+        } else {
+          // a piece of a unit split between CTAs: its normalised partial goes
+          // to the CTA's slot (0: the CTA's first piece, 1: its last piece);
+          // attn_combine_kernel merges the unit's pieces
+          const int which = (x - n == x_begin) ? 0 : 1;
+          const size_t pr = ((size_t)b * p.bnd.slots + 2 * ph + which) * UROWS + t * BM + row;
+          // O_p in bf16 (half the bytes the merge reads back), LSE_p in fp32;
+          // the LSE is kept in L2 (evict_last) until the merge reads it
+          const uint64_t pol = l2_policy_evict_last();
+          uint4* dst = reinterpret_cast<uint4*>(p.part_o + pr * HD);
+  #pragma unroll
           for (int c8 = 0; c8 < 8; ++c8) {
             uint4 w;
             w.x = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 0]) * inv_l, __uint_as_float(orr[c8 * 8 + 1]) * inv_l);
@@ -501,28 +530,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             w.w = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 6]) * inv_l, __uint_as_float(orr[c8 * 8 + 7]) * inv_l);
             dst[c8] = w;
           }
-          p.lse[(size_t)th * p.N + q] = lse_val;
+          st_global_hint(p.part_lse + pr, lse_val, pol);
         }
-      } else {
-        // a piece of a unit split between CTAs: its normalised partial goes
-        // to the CTA's slot (0: the CTA's first piece, 1: its last piece);
-        // attn_combine_kernel merges the unit's pieces
-        const int which = (x - n == x_begin) ? 0 : 1;
-        const size_t pr = ((size_t)b * 2 + which) * UROWS + t * BM + row;
-        // O_p in bf16 (half the bytes the merge reads back), LSE_p in fp32;
-        // the LSE is kept in L2 (evict_last) until the merge reads it
-        const uint64_t pol = l2_policy_evict_last();
-        uint4* dst = reinterpret_cast<uint4*>(p.part_o + pr * HD);
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          uint4 w;
-          w.x = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 0]) * inv_l, __uint_as_float(orr[c8 * 8 + 1]) * inv_l);
-          w.y = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 2]) * inv_l, __uint_as_float(orr[c8 * 8 + 3]) * inv_l);
-          w.z = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 4]) * inv_l, __uint_as_float(orr[c8 * 8 + 5]) * inv_l);
-          w.w = pack_bf16x2(__uint_as_float(orr[c8 * 8 + 6]) * inv_l, __uint_as_float(orr[c8 * 8 + 7]) * inv_l);
-          dst[c8] = w;
-        }
-        st_global_hint(p.part_lse + pr, lse_val, pol);
       }
     }
   }
@@ -548,7 +557,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 // at once, and the SMs without a merge block are free for the next kernel.
 constexpr int CMB_THREADS = 4 * BM;
 struct CombineJobs {
-  unsigned short j[2 * kAttnMaxGrid];
+  unsigned short j[2 * kAttnMaxPhases * kAttnMaxGrid];
 };
 
 __global__ void __launch_bounds__(CMB_THREADS, 2)
@@ -566,7 +575,8 @@ Params make_params(const AttnArgs& a) {
     const int nb = (a.M + BN - 1) / BN, nf = (a.N + BN - 1) / BN;
     const long long units = attn_units((a.N + BM - 1) / BM, a.H);
     const long long total = units * (nb + nf);
-    attn_split_bounds(p.bnd, units, nb, nf, (int)(a.grid < total ? a.grid : total));
+    attn_split_bounds(p.bnd, units, nb, nf, (int)(a.grid < total ? a.grid : total), a.H,
+                      (a.N + BM - 1) / BM, a.M, a.max_phases);
   }
   p.N = a.N;
   p.H = a.H;
@@ -647,7 +657,7 @@ cudaError_t launch_attention(const AttnArgs& a, cudaStream_t s, cudaEvent_t ev_b
     const SplitLayout lay = attn_split_layout(a);
     CombineJobs jobs;
     unsigned n = 0;
-    for (int j = 0; j < 2 * (a.grid - 1); ++j)
+    for (int j = 0; j < split::job_count(lay); ++j)
       if (split::job_live(lay, j)) jobs.j[n++] = (unsigned short)j;
     if (n == 0) jobs.j[n++] = 0xFFFF;  // one block that merges nothing: the launch is counted
     e = launch_pdl(attn_combine_kernel, dim3(n), dim3(CMB_THREADS), 0, s, lay, jobs);

@@ -39,24 +39,37 @@ constexpr int kStatusSmemAlign = 2;  // dynamic shared memory not 1 KB aligned
 // pieces per unit.
 constexpr int kAttnMaxGrid = 256;
 
-// The attention's stream-K split: CTA b takes key tiles [x[b], x[b + 1]) of
-// the (unit, key tile) sequence.  The cuts equalise an estimated cost, not
-// the tile count: a frame tile (the frame's own K/V, gathered from the
-// token-major frame tensor, the last one ragged) costs more than a bank
-// tile, and every unit a CTA starts costs a pipeline drain and refill.  The
-// weights are per-CTA timings of the kernel at 16.7k keys regressed on
-// these counts (a unit start ~1.7 tiles, a frame tile ~1.08).
+// The attention's stream-K split.  The (unit, key tile) sequence runs in P
+// phases (P = 1 or 2), each a contiguous run of whole head-pair groups of
+// units; CTA b takes key tiles [x[p][b], x[p][b + 1]) of phase p, phase by
+// phase.  With two phases only half of the heads' K/V is read at any time:
+// a long bank that L2 cannot hold whole (16 heads x 29,360 rows = 120 MB
+// at the 2000-frame stream's end) is otherwise re-read ~4x from HBM,
+// because the CTAs sweep every head's rows at scattered positions at once.
+//
+// The cuts equalise an estimated cost, not the tile count: a frame tile
+// (the frame's own K/V, gathered from the token-major frame tensor, the last
+// one ragged) costs more than a bank tile, and every unit a CTA starts costs
+// a pipeline drain and refill.  The weights are per-CTA timings of the
+// kernel at 16.7k keys regressed on these counts (a unit start ~1.7 tiles, a
+// frame tile ~1.08).
 constexpr int kCostBankTile = 100, kCostFrameTile = 108, kCostUnitStart = 170;
+constexpr int kAttnMaxPhases = 2;
+// K/V bytes of a launch above which it runs in two phases.
+constexpr long long kAttnPhaseKvBytes = 80ll << 20;
 struct SplitBounds {
-  long long x[kAttnMaxGrid + 1];
+  int P;                                          // phases
+  int slots;                                      // partial slots per CTA (2 x the phases allowed)
+  long long pbeg[kAttnMaxPhases + 1];             // first tile of each phase; pbeg[P] = total
+  long long x[kAttnMaxPhases][kAttnMaxGrid + 1];  // the cuts of each phase
 };
-// Cuts `units` units of nb bank tiles followed by nf frame tiles into G
-// ranges of about equal cost (1 <= G <= units * (nb + nf)): strictly
-// increasing, x[0] = 0, x[G] = units * (nb + nf).
-inline void attn_split_bounds(SplitBounds& sb, long long units, int nb, int nf, int G) {
-  const long long nkv = nb + nf, total = units * nkv;
+// Cuts units [u0, u1) (nb bank tiles then nf frame tiles each) into G ranges
+// of about equal cost, into x[0..G]: strictly increasing, x[0] = u0 (nb +
+// nf), x[G] = u1 (nb + nf).  Needs (u1 - u0) (nb + nf) >= G.
+inline void attn_cut_phase(long long* x, long long u0, long long u1, int nb, int nf, int G) {
+  const long long nkv = nb + nf, t0 = u0 * nkv, t1 = u1 * nkv;
   const long long wu = kCostUnitStart + (long long)kCostBankTile * nb + (long long)kCostFrameTile * nf;
-  const long long wt = units * wu;
+  const long long wt = (u1 - u0) * wu;
   for (int b = 0; b <= G; ++b) {
     const long long target = wt / G * b + (wt % G) * b / G;  // floor(wt b / G) without overflow
     const long long u = target / wu;
@@ -64,14 +77,41 @@ inline void attn_split_bounds(SplitBounds& sb, long long units, int nb, int nf, 
     if (r <= 0) j = 0;
     else if (r < (long long)kCostBankTile * nb) j = (r + kCostBankTile / 2) / kCostBankTile;
     else j = nb + (r - (long long)kCostBankTile * nb + kCostFrameTile / 2) / kCostFrameTile;
-    sb.x[b] = u * nkv + (j < nkv ? j : nkv);
+    x[b] = t0 + u * nkv + (j < nkv ? j : nkv);
   }
-  sb.x[0] = 0;
-  sb.x[G] = total;
+  x[0] = t0;
+  x[G] = t1;
   for (int b = 1; b < G; ++b)  // every CTA at least one tile
-    if (sb.x[b] <= sb.x[b - 1]) sb.x[b] = sb.x[b - 1] + 1;
+    if (x[b] <= x[b - 1]) x[b] = x[b - 1] + 1;
   for (int b = G - 1; b > 0; --b)
-    if (sb.x[b] > total - (G - b)) sb.x[b] = total - (G - b);
+    if (x[b] > t1 - (G - b)) x[b] = t1 - (G - b);
+}
+// The split of `units` units (H heads, nqt query tiles per head; unit order
+// of unit_tiles) over G CTAs: two phases when the K/V of the launch
+// (H M 256 bytes) exceed kAttnPhaseKvBytes, there are at least two
+// head-pair groups, max_phases allows it and each phase has at least G
+// tiles; one phase otherwise.
+inline void attn_split_bounds(SplitBounds& sb, long long units, int nb, int nf, int G, int H,
+                              int nqt, long long M, int max_phases) {
+  const long long nkv = nb + nf, total = units * nkv;
+  const long long gs = 2 * (nqt >> 1) + (nqt & 1);  // units of a two-head group
+  const long long ngroups = (H + 1) / 2;
+  sb.P = 1;
+  sb.slots = 2 * (max_phases > 1 ? kAttnMaxPhases : 1);
+  sb.pbeg[0] = 0;
+  if (max_phases > 1 && ngroups >= 2 && (long long)H * M * 256 > kAttnPhaseKvBytes) {
+    const long long u1 = ((ngroups + 1) / 2) * gs;  // whole two-head groups in phase 0
+    if (u1 * nkv >= G && (units - u1) * nkv >= G) {
+      sb.P = 2;
+      sb.pbeg[1] = u1 * nkv;
+      sb.pbeg[2] = total;
+      attn_cut_phase(sb.x[0], 0, u1, nb, nf, G);
+      attn_cut_phase(sb.x[1], u1, units, nb, nf, G);
+      return;
+    }
+  }
+  sb.pbeg[1] = total;
+  attn_cut_phase(sb.x[0], 0, units, nb, nf, G);
 }
 
 // The split as the merge of split units needs it (split.cuh).
@@ -82,8 +122,8 @@ struct SplitLayout {
   int nkv;                // key tiles per unit
   int nqt;                // query tiles per head
   int N, H;
-  const __nv_bfloat16* part_o;  // [G][2][kUnitRows][64] piece partials (bf16)
-  const float* part_lse;  // [G][2][kUnitRows]
+  const __nv_bfloat16* part_o;  // [G][bnd.slots][kUnitRows][64] piece partials (bf16)
+  const float* part_lse;  // [G][bnd.slots][kUnitRows]
   __nv_bfloat16* out;     // [N][H][64]
   float* lse;             // [H][N]
 };
@@ -98,8 +138,9 @@ struct AttnArgs {
   float scale;
   __nv_bfloat16* out;       // [N][H][64]
   float* lse;               // [H][N]
-  __nv_bfloat16* part_o;    // [grid][2][kUnitRows][64] split-piece partial outputs (bf16)
-  float* part_lse;          // [grid][2][kUnitRows]
+  __nv_bfloat16* part_o;    // [grid][2 max_phases][kUnitRows][64] split-piece partials (bf16)
+  float* part_lse;          // [grid][2 max_phases][kUnitRows]
+  int max_phases;           // 1 or 2 (kAttnMaxPhases): phases the partial scratch allows
   int* status;
   int grid;                 // CTAs of the attention kernel (<= plan.total)
   // optional launch clock (nullptr: off), this launch's words, global timer
@@ -161,9 +202,14 @@ struct AttnPlan {
 };
 AttnPlan attn_plan(int N, int H, int M);
 
-// Scratch sizes for a given grid.
-inline size_t attn_part_o_elems(int grid) { return (size_t)grid * 2 * kUnitRows * kHeadDim; }
-inline size_t attn_part_lse_floats(int grid) { return (size_t)grid * 2 * kUnitRows; }
+// Scratch sizes for a given grid and phases allowed (two partial slots per
+// CTA and phase: its first and its last piece).
+inline size_t attn_part_o_elems(int grid, int max_phases) {
+  return (size_t)grid * 2 * max_phases * kUnitRows * kHeadDim;
+}
+inline size_t attn_part_lse_floats(int grid, int max_phases) {
+  return (size_t)grid * 2 * max_phases * kUnitRows;
+}
 
 // The split of an attention launch with these arguments.
 SplitLayout attn_split_layout(const AttnArgs& a);

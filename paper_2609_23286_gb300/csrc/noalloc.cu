@@ -183,6 +183,7 @@ extern "C" REGMEM_API regmem_status regmem_attend_frame_noalloc(const regmem_fra
   a.lse = sc->lse;
   a.part_o = sc->part_o;
   a.part_lse = sc->part_lse;
+  a.max_phases = 1;  // the fixed scratch holds two partial slots per CTA
   a.status = st;
   a.wait_ns = 2000000000ull;  // 2 s
   a.fault_skip_kv = -1;

@@ -283,6 +283,7 @@ regmem_status run_attention(regmem_t* h, int layer, const void* Q, const void* K
   h->lse_layer = layer;
   a.part_o = h->part_o;
   a.part_lse = h->part_lse;
+  a.max_phases = kAttnMaxPhases;
   a.status = h->status_dev;
   a.wait_ns = h->wait_ns;
   a.fault_skip_kv = h->fault_skip_kv;
@@ -454,8 +455,8 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   RM_CUDA(h, cudaMalloc(&h->lse, (size_t)h->layers * h->heads * N * sizeof(float)));
   RM_CUDA(h, cudaMalloc(&h->qidx, q.size() * sizeof(int) + 4));
   RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
-  RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_elems(h->attn_grid) * sizeof(__nv_bfloat16)));
-  RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid) * sizeof(float)));
+  RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_elems(h->attn_grid, kAttnMaxPhases) * sizeof(__nv_bfloat16)));
+  RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid, kAttnMaxPhases) * sizeof(float)));
   RM_CUDA(h, cudaMalloc(&h->head_done, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMemset(h->head_done, 0, h->heads * sizeof(int)));
   RM_CUDA(h, cudaMalloc(&h->adm_lists, (size_t)h->heads * ((N + kTile - 1) / kTile) * 32 * sizeof(uint64_t)));

@@ -1,13 +1,13 @@
 // The attention's stream-K split and the merge of units cut between CTAs.
 //
 // The (unit, key tile) sequence -- a unit is a pair of 128-row query tiles
-// (unit_tiles), run over every key tile of [bank ; frame] -- is cut into G
-// contiguous ranges of about equal cost (attn_split_bounds), CTA b taking
-// [x[b], x[b + 1]).  A unit cut
-// by a CTA boundary leaves, from each CTA that holds part of it, one
-// normalised partial per query row, (O_p, LSE_p), in the CTA's slot 0 (the
-// unit is the CTA's first piece) or 1 (its last piece), O_p in bf16 and LSE_p
-// in fp32.  The merge of Eq. 3
+// (unit_tiles), run over every key tile of [bank ; frame] -- runs in one or
+// two phases, each cut into G contiguous ranges of about equal cost
+// (attn_split_bounds), CTA b taking [x[p][b], x[p][b + 1]) in phase p.  A
+// unit cut by a CTA boundary leaves, from each CTA that holds part of it, one
+// normalised partial per query row, (O_p, LSE_p), in the CTA's slot 2p (the
+// unit is the CTA's first piece of phase p) or 2p + 1 (its last piece), O_p in
+// bf16 and LSE_p in fp32.  The merge of Eq. 3
 // over the pieces is the log-sum-exp combination
 //     LSE = log sum_p exp(LSE_p),   O = sum_p exp(LSE_p - LSE) O_p,
 // folded in CTA order, so the result does not depend on which CTA finished
@@ -31,25 +31,27 @@ constexpr int kPrefetch = 2;            // pieces whose loads are issued togethe
 
 using Layout = SplitLayout;
 
-__host__ __device__ __forceinline__ long long range_begin(const SplitBounds& sb, int b) {
-  return sb.x[b];
+// Phase of tile x.
+__host__ __device__ __forceinline__ int phase_of(const SplitBounds& sb, long long x) {
+  return sb.P > 1 && x >= sb.pbeg[1] ? 1 : 0;
 }
 
-// CTA whose range contains tile x (binary search of the cuts).
-__host__ __device__ __forceinline__ int cta_of(const SplitBounds& sb, int G, long long x) {
-  int lo = 0, hi = G - 1;  // sb.x[lo] <= x < sb.x[hi + 1]
+// CTA whose range of phase p contains tile x (binary search of the cuts).
+__host__ __device__ __forceinline__ int cta_of(const SplitBounds& sb, int p, int G, long long x) {
+  int lo = 0, hi = G - 1;  // sb.x[p][lo] <= x < sb.x[p][hi + 1]
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    if (sb.x[mid] <= x) lo = mid;
+    if (sb.x[p][mid] <= x) lo = mid;
     else hi = mid - 1;
   }
   return lo;
 }
 
-// The CTAs holding a split unit: b_lo .. b_hi, and the slot of b_lo's piece
-// (every later CTA holds the unit as its first piece, slot 0).
+// The CTAs holding a split unit of phase p: b_lo .. b_hi, and the slot of
+// b_lo's piece (every later CTA holds the unit as its first piece of the
+// phase, slot 2p).
 struct Pieces {
-  int b_lo, b_hi, which_lo;
+  int b_lo, b_hi, which_lo, p, slots;
 };
 
 // Row `r` (0..255 within the unit) of piece i (0-based from b_lo) in the
@@ -57,7 +59,7 @@ struct Pieces {
 __device__ __forceinline__ size_t piece_row(const Pieces& pc, int i, int r) {
   const int bb = pc.b_lo + i;
   const int which = i == 0 ? pc.which_lo : 0;
-  return ((size_t)bb * 2 + which) * kUnitRowsS + r;
+  return ((size_t)bb * pc.slots + 2 * pc.p + which) * kUnitRowsS + r;
 }
 
 // Merges 16 channels (quarter qtr) of row r of tile t of split unit u and
@@ -132,8 +134,9 @@ __device__ __forceinline__ void merge_row(const Layout& s, const Pieces& pc, int
   if (qtr == 0) s.lse[(size_t)h * s.N + q] = m + __logf(den);
 }
 
-// Merge job j (0 .. 2 (G - 1) - 1): query tile j & 1 of the unit cut by the
-// boundary between CTAs j / 2 and j / 2 + 1, unless that boundary is not
+// Merge job j (0 .. 2 P (G - 1) - 1) of phase p = j / (2 (G - 1)), with
+// jj = j mod 2 (G - 1): query tile jj & 1 of the unit cut by the phase's
+// boundary between CTAs jj / 2 and jj / 2 + 1, unless that boundary is not
 // strictly inside a unit or an earlier boundary cuts the same unit.
 // prepare_job needs only the layout (it can run before the attention's
 // partials are complete); run_job merges every row of the tile with a group
@@ -143,26 +146,30 @@ struct Job {
   Pieces pc;
 };
 // Whether job j merges anything (host and device).
+__host__ __device__ inline int job_count(const Layout& s) { return 2 * s.bnd.P * (s.G - 1); }
 __host__ __device__ inline bool job_live(const Layout& s, int j) {
-  const int bnd = j / 2 + 1;
-  const long long xb = range_begin(s.bnd, bnd);
-  const int u = (int)(xb / s.nkv);
-  const long long x0 = (long long)u * s.nkv;
-  if (xb == x0 || range_begin(s.bnd, bnd - 1) > x0) return false;
-  return (j & 1) == 0 || unit_tiles(u, s.nqt, s.H).has1;
+  const int p = j / (2 * (s.G - 1)), jj = j - p * 2 * (s.G - 1);
+  const int bnd = jj / 2 + 1;
+  const long long xb = s.bnd.x[p][bnd];
+  const long long u = xb / s.nkv;
+  const long long x0 = u * s.nkv;
+  if (xb == x0 || s.bnd.x[p][bnd - 1] > x0) return false;
+  return (jj & 1) == 0 || unit_tiles(u, s.nqt, s.H).has1;
 }
 __device__ __forceinline__ Job prepare_job(const Layout& s, int j) {
   Job jb;
   jb.u = -1;
   jb.t = j & 1;
-  if (j < 0 || !job_live(s, j)) return jb;
-  const int bnd = j / 2 + 1;
-  const long long x0 = range_begin(s.bnd, bnd) / s.nkv * s.nkv;
-  const int u = (int)(x0 / s.nkv);
-  jb.u = u;
+  if (j < 0 || j >= job_count(s) || !job_live(s, j)) return jb;
+  const int p = j / (2 * (s.G - 1)), jj = j - p * 2 * (s.G - 1);
+  const int bnd = jj / 2 + 1;
+  const long long x0 = s.bnd.x[p][bnd] / s.nkv * s.nkv;
+  jb.u = (int)(x0 / s.nkv);
+  jb.pc.p = p;
+  jb.pc.slots = s.bnd.slots;
   jb.pc.b_lo = bnd - 1;  // the CTA holding the unit's first tile
-  jb.pc.b_hi = cta_of(s.bnd, s.G, x0 + s.nkv - 1);
-  jb.pc.which_lo = range_begin(s.bnd, jb.pc.b_lo) == x0 ? 0 : 1;
+  jb.pc.b_hi = cta_of(s.bnd, p, s.G, x0 + s.nkv - 1);
+  jb.pc.which_lo = s.bnd.x[p][jb.pc.b_lo] == x0 ? 0 : 1;
   return jb;
 }
 template <int NT>

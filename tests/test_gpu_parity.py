@@ -135,6 +135,7 @@ def test_teacher_forced_bank_lengths(M):
                            # tiles, head 2's last tile is a unit by itself
     (2, 1, 8, 8, 30000),   # one query tile per head: a single two-head unit over the grid
     (4, 5, 37, 37, 12000),  # two two-head units, each split over many CTAs
+    (4, 5, 8, 8, 90000),   # K/V of 92 MB: two phases (heads 0-1, then 2-3), each unit over every CTA
 ])
 def test_split_units_across_many_ctas(H, ns, gh, gw, M):
     """Few heads and a long bank: units whose key tiles are spread over many

@@ -88,18 +88,32 @@ SPLIT_PROGRAM = r"""
 #include "split.cuh"
 using namespace regmem_dev;
 int main() {
-  // (units, bank tiles, frame tiles, CTAs)
-  const int cases[][4] = {{88, 121, 11, 152}, {88, 0, 11, 152}, {88, 11, 11, 152}, {88, 230, 11, 152},
-                          {1, 313, 1, 152}, {1, 159, 1, 152}, {1, 1, 1, 2}, {3, 40, 11, 152},
-                          {8, 2, 1, 24}, {88, 2148, 11, 256}, {5, 0, 3, 15}};
+  // (heads, query tiles per head, bank rows M, frame tiles, CTAs, phases allowed)
+  const long long cases[][6] = {{16, 11, 15486, 11, 152, 2}, {16, 11, 0, 11, 152, 2},
+                                {16, 11, 1374, 11, 152, 2}, {16, 11, 29360, 11, 152, 2},
+                                {16, 11, 29360, 11, 152, 1}, {1, 1, 40000, 1, 152, 2},
+                                {1, 1, 20352, 1, 152, 2}, {2, 1, 1, 1, 2, 2}, {3, 11, 5000, 11, 152, 2},
+                                {4, 1, 90000, 1, 152, 2}, {4, 11, 12000, 11, 152, 2},
+                                {16, 11, 274800, 11, 256, 2}, {5, 9, 0, 9, 15, 2}, {7, 3, 70000, 3, 152, 2}};
   for (const auto& c : cases) {
+    const int H = (int)c[0], nqt = (int)c[1], nf = (int)c[3], G = (int)c[4], mp = (int)c[5];
+    const long long M = c[2];
+    const int nb = (int)((M + 127) / 128);
+    const long long units = attn_units(nqt, H);
     SplitBounds sb;
-    attn_split_bounds(sb, c[0], c[1], c[2], c[3]);
-    std::printf("case %d %d %d %d\n", c[0], c[1], c[2], c[3]);
-    for (int b = 0; b <= c[3]; ++b) std::printf("%lld ", sb.x[b]);
+    attn_split_bounds(sb, units, nb, nf, G, H, nqt, M, mp);
+    std::printf("case %d %d %lld %d %d %d %lld %d %d\n", H, nqt, M, nf, G, mp, units, sb.P, sb.slots);
+    for (int p = 0; p <= sb.P; ++p) std::printf("%lld ", sb.pbeg[p]);
     std::printf("\n");
-    const long long total = (long long)c[0] * (c[1] + c[2]);
-    for (long long x = 0; x < total; x += 1 + total / 997) std::printf("%lld:%d ", x, split::cta_of(sb, c[3], x));
+    for (int p = 0; p < sb.P; ++p) {
+      for (int b = 0; b <= G; ++b) std::printf("%lld ", sb.x[p][b]);
+      std::printf("\n");
+    }
+    const long long total = units * (nb + nf);
+    for (long long x = 0; x < total; x += 1 + total / 997) {
+      const int p = split::phase_of(sb, x);
+      std::printf("%lld:%d:%d ", x, p, split::cta_of(sb, p, G, x));
+    }
     std::printf("\n");
   }
   return 0;
@@ -108,10 +122,13 @@ int main() {
 
 
 def test_weighted_split_covers_every_tile_once_and_balances_cost(tmp_path):
-    """attn_split_bounds cuts the (unit, key tile) sequence into G ranges:
-    strictly increasing, from 0 to units * (nb + nf), each CTA's estimated
-    cost (bank tile 100, frame tile 108, a unit start 170) within one tile
-    and one unit start of the mean; cta_of inverts the cuts."""
+    """attn_split_bounds cuts the (unit, key tile) sequence into G ranges per
+    phase: strictly increasing, each phase a run of whole head-pair groups of
+    units, the phases together from 0 to units * (nb + nf), each CTA's
+    estimated cost (bank tile 100, frame tile 108, a unit start 170) within
+    one tile and one unit start of the phase's mean; two phases exactly when
+    the K/V bytes H M 256 exceed 80 MB, there are two head-pair groups and two
+    phases are allowed; phase_of / cta_of invert the cuts."""
     nvcc = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
     if not os.path.exists(nvcc):
         pytest.skip("nvcc not found")
@@ -120,22 +137,36 @@ def test_weighted_split_covers_every_tile_once_and_balances_cost(tmp_path):
     subprocess.run([nvcc, "-std=c++17", "-I", CSRC, "-I", os.path.join(ROOT, "include"),
                     str(src), "-o", str(exe)], check=True, capture_output=True)
     lines = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.splitlines()
-    for i in range(0, len(lines), 3):
-        units, nb, nf, G = map(int, lines[i].split()[1:])
-        x = list(map(int, lines[i + 1].split()))
+    i = 0
+    seen_two = 0
+    while i < len(lines):
+        H, nqt, M, nf, G, mp, units, P, slots = map(int, lines[i].split()[1:])
+        nb = -(-M // 128)
         nkv, total = nb + nf, units * (nb + nf)
-        assert len(x) == G + 1 and x[0] == 0 and x[-1] == total
-        assert all(a < b for a, b in zip(x, x[1:]))
-        cost = []
-        for b in range(G):
-            c = 0
-            for t in range(x[b], x[b + 1]):
-                j = t % nkv
-                c += (170 if j == 0 else 0) + (100 if j < nb else 108)
-            cost.append(c)
-        mean = sum(cost) / G
-        if total >= 4 * G:  # enough tiles per CTA for the cut to balance cost
-            assert max(cost) - mean <= 108 + 170 and mean - min(cost) <= 108 + 170, (units, nb, nf, G)
-        for pair in lines[i + 2].split():
-            t, b = map(int, pair.split(":"))
-            assert x[b] <= t < x[b + 1]
+        gs = 2 * (nqt // 2) + (nqt % 2)
+        pbeg = list(map(int, lines[i + 1].split()))
+        cuts = [list(map(int, lines[i + 2 + p].split())) for p in range(P)]
+        want_two = mp > 1 and (H + 1) // 2 >= 2 and H * M * 256 > 80 * 2 ** 20
+        assert P == (2 if want_two else 1) and slots == (4 if mp > 1 else 2)
+        seen_two += P == 2
+        assert pbeg[0] == 0 and pbeg[-1] == total
+        for p in range(P):
+            x = cuts[p]
+            assert len(x) == G + 1 and x[0] == pbeg[p] and x[-1] == pbeg[p + 1]
+            assert pbeg[p] % (gs * nkv) == 0  # phases begin at head-pair groups
+            assert all(a < b for a, b in zip(x, x[1:]))
+            cost = []
+            for b in range(G):
+                c = 0
+                for t in range(x[b], x[b + 1]):
+                    j = t % nkv
+                    c += (170 if j == 0 else 0) + (100 if j < nb else 108)
+                cost.append(c)
+            mean = sum(cost) / G
+            if pbeg[p + 1] - pbeg[p] >= 4 * G:  # enough tiles per CTA to balance cost
+                assert max(cost) - mean <= 108 + 170 and mean - min(cost) <= 108 + 170, lines[i]
+        for trip in lines[i + 2 + P].split():
+            t, p, b = map(int, trip.split(":"))
+            assert pbeg[p] <= t < pbeg[p + 1] and cuts[p][b] <= t < cuts[p][b + 1]
+        i += 3 + P
+    assert seen_two >= 3
