@@ -762,9 +762,10 @@ def main(argv=None):
     ap.add_argument("--layers", type=int, default=0, help="override the config's layer count")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--overlap", type=int, choices=[0, 1], default=1,
+    ap.add_argument("--overlap", type=int, choices=[0, 1], default=None,
                     help="1: saliency and admission on the library's side stream, overlapping "
-                         "the next layer's attention")
+                         "the next layer's attention (default: 1 with several layers; 0 for a "
+                         "single layer, whose next attention always waits for that side work)")
     ap.add_argument("--two-call", action="store_true",
                     help="per layer regmem_attend_frame + regmem_admit instead of regmem_attend_admit")
     ap.add_argument("--frames", type=int, default=0, help="override the config's stream length")
@@ -786,6 +787,8 @@ def main(argv=None):
     cfg = dict(CONFIGS[args.config])
     if args.layers:
         cfg["layers"] = args.layers
+    if args.overlap is None:
+        args.overlap = 1 if cfg["layers"] > 1 else 0
     if args.frames:
         cfg["frames"] = args.frames
     variant = {}
