@@ -30,7 +30,8 @@ Also reported:
                 sustained for longer ones)
   e2e           same metric through regmem_attend_admit_host: pinned host
                 Q/K/V in, O and saliency back to host, copies inside the timed
-                region
+                region; the window is timed three times (banks restored
+                between, untimed) and the value is all frames / all time
   cpu_baseline  the fp64 oracle on the host cores, timed on a bounded sample
                 of the same frames (single layer-frames at the window's ends,
                 cost linear in the attended length)
@@ -131,6 +132,9 @@ def bench_config(cfg, name, S0, K, world):
 # roofline itself comes from the attention's launch clock, which times every
 # launch without events.
 PROFILE_EVERY = 61
+
+# Times the e2e leg runs the timed window (value: all frames / all time).
+E2E_REPS = 3
 
 
 def describe(cfg, name):
@@ -552,23 +556,31 @@ def gpu_arm(args, cfg, cfg_name):
         rm.profile_enable(0)
         host_frames(S0, W)
         rm.synchronize()
-        restore()
-        barrier()
-        torch.cuda.synchronize()
-        # host clock around the calls and the final synchronisation: the
-        # library's copies run on a stream of its own
-        t_e0 = time.perf_counter()
-        host_frames(S0, K)
-        t_enq = time.perf_counter()
-        rm.synchronize()
-        e2e_ms = max_over_ranks((time.perf_counter() - t_e0) * 1e3, dev)
-        enqueue_ms = (t_enq - t_e0) * 1e3
+        # the window is timed E2E_REPS times (banks restored, untimed, in
+        # between): one short window's host-to-device copies are exposed to
+        # whatever else the host does at that moment
+        rep_ms, enqueue_ms = [], 0.0
+        for _ in range(E2E_REPS):
+            restore()
+            barrier()
+            torch.cuda.synchronize()
+            # host clock around the calls and the final synchronisation: the
+            # library's copies run on a stream of its own
+            t_e0 = time.perf_counter()
+            host_frames(S0, K)
+            t_enq = time.perf_counter()
+            rm.synchronize()
+            rep_ms.append((time.perf_counter() - t_e0) * 1e3)
+            enqueue_ms += (t_enq - t_e0) * 1e3
+        e2e_ms = max_over_ranks(sum(rep_ms), dev)
         barrier()
         tb = N * H * 64 * 2
-        e2e = {"value": round(K * world / (e2e_ms / 1e3), 3), "unit": UNIT,
+        e2e = {"value": round(E2E_REPS * K * world / (e2e_ms / 1e3), 3), "unit": UNIT,
                "h2d_bytes_per_step": 3 * tb * L, "d2h_bytes_per_step": (tb + H * N * 4) * L,
                "api": "regmem_attend_admit_host (pinned host buffers)",
-               "host_enqueue_ms_per_step": round(enqueue_ms / K, 4)}
+               "repetitions_of_the_window": E2E_REPS,
+               "repetition_values": [round(K * world / (m / 1e3), 3) for m in rep_ms],
+               "host_enqueue_ms_per_step": round(enqueue_ms / (E2E_REPS * K), 4)}
 
     launches = int(sum_over_ranks(prof.launches(), dev))
     rm.close()
