@@ -55,7 +55,11 @@ typedef enum regmem_status {
   REGMEM_ERR_CAPACITY = -3,    /* admission would overflow the bank          */
   REGMEM_ERR_CUDA = -4,        /* CUDA runtime / driver error                */
   REGMEM_ERR_UNSUPPORTED = -5, /* shape outside what the kernels handle      */
-  REGMEM_ERR_TIMEOUT = -6      /* a device-side bounded wait expired         */
+  REGMEM_ERR_TIMEOUT = -6,     /* a device-side bounded wait expired         */
+  REGMEM_ERR_DEVICE_CHECK = -7 /* a range guard of the checked build failed:
+                                  libregmem_checked.so, compiled with
+                                  REGMEM_DEVICE_CHECKS, checks the indices its
+                                  kernels derive before global accesses      */
 } regmem_status;
 
 /* Frame geometry.  Tokens of a frame are ordered [special tokens, patch tokens

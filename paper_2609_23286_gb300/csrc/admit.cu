@@ -99,7 +99,7 @@ __global__ void __launch_bounds__(THREADS) admit_shared_kernel(AdmitArgs a) {
 
 __global__ void copy_rows_kernel(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
                                  __nv_bfloat16* bankV, long long cap, long long M, int lo, int n,
-                                 int H, int32_t* idx_out, int idx_rows) {
+                                 int H, int32_t* idx_out, int idx_rows, int n_tokens, int* status) {
   grid_dep_wait();
   grid_dep_launch();
   const long long total = (long long)n * H * 8;  // 16-byte chunks per tensor
@@ -111,6 +111,7 @@ __global__ void copy_rows_kernel(const __nv_bfloat16* K, const __nv_bfloat16* V,
     const long long rh = e >> 3;  // r * H + h
     const int h = (int)(rh % H);
     const long long r = rh / H;
+    if (!dev_check(lo + r < n_tokens && M + r < cap, status)) continue;
     const uint4* src = reinterpret_cast<const uint4*>((which ? V : K) + ((lo + r) * H + h) * HD);
     uint4* dst = reinterpret_cast<uint4*>((which ? bankV : bankK) + ((size_t)h * cap + M + r) * HD);
     dst[c] = src[c];
@@ -121,12 +122,13 @@ __global__ void copy_rows_kernel(const __nv_bfloat16* K, const __nv_bfloat16* V,
 // idx_out (optional) receives lo + r for r < n, in `idx_rows` rows of n.
 cudaError_t launch_copy_rows(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
                              __nv_bfloat16* bankV, long long cap, long long M, int lo, int n, int H,
-                             int32_t* idx_out, int idx_rows, cudaStream_t s) {
+                             int32_t* idx_out, int idx_rows, int n_tokens, int* status,
+                             cudaStream_t s) {
   const long long work = 2LL * n * H * 8;
   int blocks = (int)((work + 255) / 256);
   if (blocks > 4096) blocks = 4096;
   return launch_pdl(copy_rows_kernel, dim3(blocks), dim3(256), 0, s, K, V, bankK, bankV, cap, M, lo, n,
-                    H, idx_out, idx_rows);
+                    H, idx_out, idx_rows, n_tokens, status);
 }
 
 }  // namespace
@@ -144,7 +146,8 @@ cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s) {
   if (nc < 1 || nc > kMaxCandidates || a.k < 0 || a.k > nc) return cudaErrorInvalidValue;
   if (a.k == 0) return cudaSuccess;
   if (a.k == nc)  // every candidate: nothing to rank
-    return launch_copy_rows(a.K, a.V, a.bankK, a.bankV, a.cap, a.M, a.cand_lo, nc, a.H, a.idx_out, a.H, s);
+    return launch_copy_rows(a.K, a.V, a.bankK, a.bankV, a.cap, a.M, a.cand_lo, nc, a.H, a.idx_out, a.H,
+                            a.N, a.status, s);
   if (a.k <= sel::kListK && a.lists && a.done) {
     const int nkt = (a.N + LT - 1) / LT;
     return launch_pdl(admit_lists_kernel, dim3(a.H * nkt), dim3(LT), 0, s, a, nkt);
@@ -157,13 +160,15 @@ cudaError_t launch_admit_shared(const AdmitArgs& a, cudaStream_t s) {
   if (nc < 1 || nc > kMaxCandidates || a.k < 0 || a.k > nc) return cudaErrorInvalidValue;
   if (a.k == 0) return cudaSuccess;
   if (a.k == nc)  // every candidate; one index list
-    return launch_copy_rows(a.K, a.V, a.bankK, a.bankV, a.cap, a.M, a.cand_lo, nc, a.H, a.idx_out, 1, s);
+    return launch_copy_rows(a.K, a.V, a.bankK, a.bankV, a.cap, a.M, a.cand_lo, nc, a.H, a.idx_out, 1,
+                            a.N, a.status, s);
   return launch_pdl(admit_shared_kernel, dim3(a.H), dim3(THREADS), (size_t)(nc + a.k) * sizeof(int), s, a);
 }
 
 cudaError_t launch_anchor(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
-                          __nv_bfloat16* bankV, long long cap, int N, int H, cudaStream_t s) {
-  return launch_copy_rows(K, V, bankK, bankV, cap, 0, 0, N, H, nullptr, 0, s);
+                          __nv_bfloat16* bankV, long long cap, int N, int H, int* status,
+                          cudaStream_t s) {
+  return launch_copy_rows(K, V, bankK, bankV, cap, 0, 0, N, H, nullptr, 0, N, status, s);
 }
 
 }  // namespace regmem_dev

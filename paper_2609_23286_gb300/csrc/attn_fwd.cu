@@ -517,6 +517,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           // attn_combine_kernel merges the unit's pieces
           const int which = (x - n == x_begin) ? 0 : 1;
           const size_t pr = ((size_t)b * p.bnd.slots + 2 * ph + which) * UROWS + t * BM + row;
+          if (!dev_check(2 * ph + which < p.bnd.slots, p.status)) continue;
           // O_p in bf16 (half the bytes the merge reads back), LSE_p in fp32;
           // the LSE is kept in L2 (evict_last) until the merge reads it
           const uint64_t pol = l2_policy_evict_last();
@@ -615,6 +616,7 @@ SplitLayout attn_split_layout(const AttnArgs& a) {
   l.part_lse = a.part_lse;
   l.out = a.out;
   l.lse = a.lse;
+  l.status = a.status;
   return l;
 }
 

@@ -34,6 +34,27 @@ constexpr int kTile = 128;      // query rows / key rows per tile
 // Bits of the device status word (written by kernels, read by the host).
 constexpr int kStatusTimeout = 1;    // a bounded wait expired
 constexpr int kStatusSmemAlign = 2;  // dynamic shared memory not 1 KB aligned
+constexpr int kStatusRange = 4;      // a range guard of the checked build failed
+
+// Range guards of the checked build (compiled with REGMEM_DEVICE_CHECKS, as
+// libregmem_checked.so): an index a kernel derives before a global access
+// is checked against its buffer; a failed check records kStatusRange in the
+// status word and the access is skipped.  In the normal build dev_check is
+// `true` and compiles away.
+#ifdef REGMEM_DEVICE_CHECKS
+constexpr bool kDeviceChecks = true;
+#else
+constexpr bool kDeviceChecks = false;
+#endif
+__device__ __forceinline__ bool dev_check(bool ok, int* status) {
+  if constexpr (kDeviceChecks) {
+    if (!ok) {
+      atomicOr(status, kStatusRange);
+      return false;
+    }
+  }
+  return true;
+}
 
 // Largest attention grid: the merge of split units lists at most this many
 // pieces per unit.
@@ -126,6 +147,7 @@ struct SplitLayout {
   const float* part_lse;  // [G][bnd.slots][kUnitRows]
   __nv_bfloat16* out;     // [N][H][64]
   float* lse;             // [H][N]
+  int* status;            // device status word (range guards of the checked build)
 };
 
 struct AttnArgs {
@@ -238,6 +260,7 @@ struct AdmitArgs {
   // per head selects alone
   uint64_t* lists;          // [H][ceil(N/128)][32]
   int* done;                // [H]
+  int* status;              // device status word (range guards of the checked build)
 };
 cudaError_t admit_setup();
 // Per-head admission (Eq. 6): k rows per head, idx_out [H][k].
@@ -247,7 +270,7 @@ cudaError_t launch_admit(const AdmitArgs& a, cudaStream_t s);
 cudaError_t launch_admit_shared(const AdmitArgs& a, cudaStream_t s);
 // First frame (Eq. 4): bank[h][0:N] = frame rows of head h.
 cudaError_t launch_anchor(const __nv_bfloat16* K, const __nv_bfloat16* V, __nv_bfloat16* bankK,
-                          __nv_bfloat16* bankV, long long cap, int N, int H, cudaStream_t s);
+                          __nv_bfloat16* bankV, long long cap, int N, int H, int* status, cudaStream_t s);
 
 // LSE-Saliency over the frame's own keys, per (head, 128-key tile).  With
 // `adm` set (1 <= k <= 32, sal == adm->sal, lists and done given), each block

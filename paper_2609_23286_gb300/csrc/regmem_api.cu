@@ -206,6 +206,10 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 regmem_status check_device_status(regmem_t* h) {
   if (h->status_host && *reinterpret_cast<volatile int*>(h->status_host) != 0) {
     const int s = *reinterpret_cast<volatile int*>(h->status_host);
+    if (s & kStatusRange)
+      return fail(h, REGMEM_ERR_DEVICE_CHECK,
+                  "a kernel reported device status 0x%x (a range guard of the checked build "
+                  "failed); destroy the handle", s);
     return fail(h, REGMEM_ERR_TIMEOUT,
                 "a kernel reported device status 0x%x (%s); destroy the handle", s,
                 (s & kStatusTimeout) ? "bounded wait expired" : "shared-memory alignment");
@@ -349,6 +353,7 @@ const char* regmem_status_string(regmem_status s) {
     case REGMEM_ERR_CUDA: return "REGMEM_ERR_CUDA";
     case REGMEM_ERR_UNSUPPORTED: return "REGMEM_ERR_UNSUPPORTED";
     case REGMEM_ERR_TIMEOUT: return "REGMEM_ERR_TIMEOUT";
+    case REGMEM_ERR_DEVICE_CHECK: return "REGMEM_ERR_DEVICE_CHECK";
   }
   return "REGMEM_UNKNOWN";
 }
@@ -589,6 +594,7 @@ AdmitArgs admit_args(regmem_t* h, int32_t layer, const void* K, const void* V, f
   a.idx_out = idx_out;
   a.lists = h->adm_lists;
   a.done = h->head_done;
+  a.status = h->status_dev;
   return a;
 }
 
@@ -656,7 +662,7 @@ regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, con
     auto* bk = h->bankK + (size_t)layer * h->heads * h->cap * kHeadDim;
     auto* bv = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
     RM_CUDA(h, launch_anchor(static_cast<const __nv_bfloat16*>(K), static_cast<const __nv_bfloat16*>(V),
-                             bk, bv, h->cap, h->N, h->heads, sst));
+                             bk, bv, h->cap, h->N, h->heads, h->status_dev, sst));
     h->prof.launches_anchor += 1;
     h->len[layer] = h->N;
     return finish_side(h, layer, sst);
@@ -774,7 +780,8 @@ regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_o
   if (h->len[layer] == 0) {  // Eq. 4: the first frame is kept whole
     auto* bk = h->bankK + (size_t)layer * h->heads * h->cap * kHeadDim;
     auto* bv = h->bankV + (size_t)layer * h->heads * h->cap * kHeadDim;
-    RM_CUDA(h, launch_anchor(h->pK[layer], h->pV[layer], bk, bv, h->cap, h->N, h->heads, h->stream));
+    RM_CUDA(h, launch_anchor(h->pK[layer], h->pV[layer], bk, bv, h->cap, h->N, h->heads, h->status_dev,
+                             h->stream));
     h->prof.launches_anchor += 1;
     h->len[layer] = h->N;
     h->pending[layer] = 0;

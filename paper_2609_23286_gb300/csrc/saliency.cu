@@ -87,6 +87,7 @@ __device__ __forceinline__ void gather_rows(const Params& p, int h, int g0, int 
   for (int c = 0; c < QS; ++c) {
     const int i = (g0 + c) * BT + tid;
     tok[c] = (g0 + c < g1 && i < p.nq) ? __ldg(p.qidx + i) : -1;
+    if (!dev_check(tok[c] < p.N, p.status)) tok[c] = -1;
   }
 #pragma unroll
   for (int c = 0; c < QS; ++c) {

@@ -294,6 +294,7 @@ __device__ __forceinline__ void append_rows(const AdmitArgs& a, int h, const int
     const int rem = w - which * a.k * 8;
     const int r = rem >> 3, c = rem & 7;
     const int tok = a.cand_lo + ord[r];
+    if (!dev_check(tok >= a.cand_lo && tok < a.N && a.M + r < a.cap, a.status)) continue;
     const __nv_bfloat16* src = (which ? a.V : a.K) + ((size_t)tok * a.H + h) * HD;
     __nv_bfloat16* dst = (which ? a.bankV : a.bankK) + ((size_t)h * a.cap + a.M + r) * HD;
     reinterpret_cast<uint4*>(dst)[c] = reinterpret_cast<const uint4*>(src)[c];

@@ -73,6 +73,7 @@ __device__ __forceinline__ void merge_row(const Layout& s, const Pieces& pc, int
   const int q = (t ? ut.qt1 : ut.qt0) * kRows + r;
   const int ur = t * kRows + r;  // row within the unit
   const int np = pc.b_hi - pc.b_lo + 1;
+  if (!dev_check(pc.b_lo >= 0 && pc.b_hi < s.G && np >= 2 && 2 * pc.p + 1 < pc.slots, s.status)) return;
   // the partials were kept in L2 for this read; afterwards they may go
   const uint64_t pol = ptx::l2_policy_evict_first();
   float lp[kPrefetch];

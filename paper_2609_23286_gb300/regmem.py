@@ -13,8 +13,11 @@ import os
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libregmem.so")
+# the same library with the kernels' range guards compiled in (build(checks=True))
+CHECKED_LIB_PATH = os.path.join(_HERE, "libregmem_checked.so")
 
 OK, ERR_ARG, ERR_STATE, ERR_CAPACITY, ERR_CUDA, ERR_UNSUPPORTED, ERR_TIMEOUT = 0, -1, -2, -3, -4, -5, -6
+ERR_DEVICE_CHECK = -7
 
 # Every exported entry point of include/regmem.h with its ctypes signature.
 _P = ctypes.c_void_p

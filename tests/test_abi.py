@@ -30,10 +30,12 @@ def test_header_declares_entry_points():
 
 
 def test_library_exports_every_declared_symbol(lib_path):
-    out = subprocess.run(["nm", "-D", "--defined-only", lib_path], capture_output=True,
-                         text=True, check=True).stdout
-    exported = sorted(set(re.findall(r"\bT (regmem_\w+)", out)))
-    assert exported == declared()
+    from paper_2609_23286_gb300 import regmem
+    for path in (lib_path, regmem.CHECKED_LIB_PATH):  # the normal and the range-checked build
+        out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True,
+                             text=True, check=True).stdout
+        exported = sorted(set(re.findall(r"\bT (regmem_\w+)", out)))
+        assert exported == declared(), path
 
 
 def test_library_loads_without_gpu_and_binding_covers_header(lib_path):
