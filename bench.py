@@ -45,6 +45,7 @@ Under torchrun with --gpus N each rank runs an independent replica stream
 from __future__ import annotations
 
 import argparse
+import gc
 import json
 import math
 import os
@@ -518,11 +519,16 @@ def gpu_arm(args, cfg, cfg_name):
     barrier()
     torch.cuda.synchronize()
     clocks.start()
+    # no collector pass of Python's own inside a timed region (a full pass
+    # can hold the enqueueing thread for tens of milliseconds)
+    gc.collect()
+    gc.disable()
     ev0.record(stream)
     run_frames(rm, cfg, pool, S0, K, out, sal, fa_out, args.two_call)
     rm.join()  # the last layers' side work ends inside the timed region
     ev1.record(stream)
     torch.cuda.synchronize()
+    gc.enable()
     barrier()
     clocks.stop()
     prof = rm.profile_read()
@@ -564,6 +570,8 @@ def gpu_arm(args, cfg, cfg_name):
             restore()
             barrier()
             torch.cuda.synchronize()
+            gc.collect()
+            gc.disable()
             # host clock around the calls and the final synchronisation: the
             # library's copies run on a stream of its own
             t_e0 = time.perf_counter()
@@ -571,6 +579,7 @@ def gpu_arm(args, cfg, cfg_name):
             t_enq = time.perf_counter()
             rm.synchronize()
             rep_ms.append((time.perf_counter() - t_e0) * 1e3)
+            gc.enable()
             enqueue_ms += (t_enq - t_e0) * 1e3
         e2e_ms = max_over_ranks(sum(rep_ms), dev)
         barrier()
