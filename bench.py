@@ -76,7 +76,7 @@ CONFIGS = {
 # {(config, attended rows L): bytes}.  The line reports the capture whose L
 # lies within 2 % of the timed launches' mean L, else null; the table is
 # emptied whenever the attention kernel changes until it is captured again.
-ATTN_TRAFFIC_CAPTURES = {("long", 16734): 73.73e6, ("long", 30720): 135.28e6}
+ATTN_TRAFFIC_CAPTURES = {("long", 16734): 73.76e6, ("long", 30720): 135.28e6}
 
 
 def traffic_for(cfg_name, mean_L):
