@@ -713,6 +713,25 @@ def gpu_arm(args, cfg, cfg_name):
             "frac": round(fa_tf / peak, 4), "launches": prof.frame_attention_clocked,
             "mean_launch_ms": round(fa_ms, 5), "algorithmic_flops_per_launch": fa_flops,
         }
+    # The paper's own figures for this path, beside ours as context (not a
+    # target): it reports no throughput and no memory measurement in its text,
+    # only the saliency's added latency (the query-downsampling sensitivity
+    # table and the head-specific retention ablation table), all on one
+    # NVIDIA RTX 3090 (24 GB, Sec. 4 implementation details), and the memory
+    # law |M_t| = |M_1| + (t - 1) floor(gamma N) of Eq. 6.
+    n_tok = cfg["ns"] + cfg["gh"] * cfg["gw"]
+    end_rows = [attended_rows(cfg, cfg["frames"] + 1, l) - n_tok for l in range(L)]
+    line["paper_context"] = {
+        "hardware": "NVIDIA RTX 3090, 24 GB",
+        "throughput_reported": None,
+        "saliency_latency_ms": {"ds 2x2 (default)": 8.29, "ds 1x1": 17.64, "ds 3x3": 7.69,
+                                "ds 4x4": 7.45, "without head-specific retention": 17.66},
+        "saliency_latency_note": "extra inference latency of the saliency estimate; precision, "
+                                 "sequence length and unit (per frame or per sequence) not stated",
+        "memory_law": "|M_t| = |M_1| + (t - 1) floor(gamma N), gamma = 0.01 (Eq. 6)",
+        "this_workload_bank_rows_per_layer_at_stream_end": max(end_rows),
+        "this_workload_bank_bytes_at_stream_end": int(sum(end_rows) * H * 64 * 2 * 2),
+    }
     if cfg.get("variant"):
         share = line["roofline"]["share_of_step"] or 0.0
         line["memory"] = {

@@ -39,3 +39,8 @@ def test_bench_json_line_tiny_stream():
     e = d["e2e"]
     assert e["value"] > 0 and e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
     assert "sm_mhz" in d["clocks"] and "reasons" in d["clocks"]
+    # the paper's figures as context, and this stream's bank at its end by the
+    # memory law of Eq. 6: 69 rows at frame 1, one per head per later frame
+    pc = d["paper_context"]
+    assert pc["hardware"].startswith("NVIDIA RTX 3090") and pc["saliency_latency_ms"]["ds 2x2 (default)"] == 8.29
+    assert pc["this_workload_bank_rows_per_layer_at_stream_end"] == 69 + 7
