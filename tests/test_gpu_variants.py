@@ -101,6 +101,50 @@ def test_unregulated_full_kv_stream(H, ns, gh, gw, frames):
         st.close()
 
 
+def test_unregulated_end_size_sampled_rows():
+    """The largest memory of the configurations: frame 200 of the unregulated
+    stream attends the 199 whole frames before it (273,426 bank rows per
+    head, 1.1 GB of K/V over 16 heads).  That launch runs in two phases, with
+    every unit spread over the whole grid.  O and LSE are checked on sampled
+    query rows of every head, the saliency on two heads (the oracle
+    materialises their 361 x 274,800 logits).  The admission of all N
+    candidates then fills the capacity exactly."""
+    H, ns, gh, gw = 16, 5, 37, 37
+    N = ns + gh * gw
+    M = 199 * N
+    st = Stream(1, H, ns, gh, gw, budget=N, max_frames=200, seed=33, candidates=1)
+    try:
+        g = torch.Generator().manual_seed(12)
+        bk = (torch.randn(H, M, 64, generator=g)
+              * torch.exp(0.5 * torch.randn(1, M, 1, generator=g))).to(torch.bfloat16)
+        bv = torch.randn(H, M, 64, generator=g).to(torch.bfloat16)
+        st.rm.import_bank(0, bk, bv, M)
+        q, k, v = st.inputs(0, 200)
+        out, sal, lse = st.attend(0, q, k, v)
+        torch.cuda.synchronize()
+        qi = orc.sampled_query_tokens(ns, gh, gw, 2)
+        rows = sorted(set(list(range(0, N, 211)) + [N - 1, 127, 128]))
+        q64, k64, v64 = to64(q), to64(k), to64(v)
+        for h in range(H):
+            kc = np.concatenate([bk[h].double().numpy(), k64[:, h]])
+            vc = np.concatenate([bv[h].double().numpy(), v64[:, h]])
+            o_r, l_r, _, _ = orc.attend_head(q64[rows, h], kc, vc, 1 / 8)
+            o_a, _, _, _ = orc.attend_head(q64[rows, h], kc, np.abs(vc), 1 / 8)
+            check_o(out[rows, h], o_r, f"h={h}", o_abs=o_a)
+            check_lse(lse[h, rows], l_r, f"h={h}")
+            if h in (0, H - 1):
+                _, l_s, z_s, _ = orc.attend_head(q64[qi, h], kc, vc, 1 / 8)
+                s_r = orc.saliency_lse(z_s, l_s, M, list(range(len(qi))))
+                check_saliency(sal[h], s_r, f"h={h}")
+                del z_s
+        idx = st.admit(0, N)
+        st.rm.synchronize()
+        assert st.rm.memory_len(0) == M + N == 200 * N
+        assert np.array_equal(idx.cpu().numpy(), np.tile(np.arange(N), (H, 1)))
+    finally:
+        st.close()
+
+
 def test_paper_layer_split_stream():
     """Sec. 4.1 / Eq. 5-6 on a 24-layer stream of small frames: layers 11-17
     admit k per frame, the others keep only the anchor frame; outputs match
