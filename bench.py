@@ -407,8 +407,9 @@ def make_pool(cfg, P, seed, device):
 
 def run_frames(rm, cfg, pool, t0, count, out, sal, fa_out=None, two_call=False):
     """Enqueue frames t0 .. t0+count-1 (all layers) through the C ABI: one
-    regmem_attend_admit per layer, or regmem_attend_frame + regmem_admit
-    (regmem_admit_shared for the head-averaged selection)."""
+    regmem_attend_admit per layer (regmem_attend_admit_shared for the
+    head-averaged selection), or with `two_call` regmem_attend_frame +
+    regmem_admit (regmem_admit_shared)."""
     P = len(pool[0])
     shared = cfg.get("selection") == "head-averaged"
     for t in range(t0, t0 + count):
@@ -418,11 +419,11 @@ def run_frames(rm, cfg, pool, t0, count, out, sal, fa_out=None, two_call=False):
             if fa_out is not None:
                 fq, fk, fv = pool[layer][t % P]
                 rm.frame_attention(fq, fk, fv, fa_out)
-            if two_call or shared:
+            if two_call:
                 rm.attend_frame(layer, q, k, v, out, sal)
                 (rm.admit_shared if shared else rm.admit)(layer, kk)
             else:
-                rm.attend_admit(layer, q, k, v, out, sal, kk)
+                (rm.attend_admit_shared if shared else rm.attend_admit)(layer, q, k, v, out, sal, kk)
 
 
 def synthetic_bank(cfg, rows, seed, device):
@@ -854,6 +855,7 @@ def main(argv=None):
     if args.head_avg:
         cfg["selection"] = "head-averaged"
         variant["selection"] = "head-averaged (one index set for all heads)"
+        args.no_e2e = True  # the host-buffer call selects per head: no e2e leg for this variant
     if variant:
         variant["k_per_layer"] = [layer_k(cfg, l) for l in range(cfg["layers"])]
         cfg["variant"] = variant

@@ -640,10 +640,15 @@ regmem_status regmem_attend_frame(regmem_t* h, int32_t layer, const void* Q, con
   return REGMEM_OK;
 }
 
-regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, const void* K,
-                                  const void* V, void* out, float* saliency, int32_t k,
-                                  int32_t* idx_out) {
-  REGMEM_RANGE;
+namespace {
+
+// regmem_attend_admit and regmem_attend_admit_shared: the attention on the
+// handle's stream, then the saliency and the selection (per head, fused into
+// the saliency kernel for k <= 32, or head-averaged) and the append on the
+// side stream when overlap is on.
+regmem_status attend_admit_impl(regmem_t* h, int32_t layer, const void* Q, const void* K,
+                                const void* V, void* out, float* saliency, int32_t k,
+                                int32_t* idx_out, bool shared) {
   regmem_status s = ready(h, layer, true);
   if (s != REGMEM_OK) return s;
   if ((s = check_tensors(h, Q, K, V, out, saliency)) != REGMEM_OK) return s;
@@ -669,17 +674,33 @@ regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, con
   }
   if ((s = check_admit(h, layer, k)) != REGMEM_OK) return s;
   const AdmitArgs a = admit_args(h, layer, K, V, saliency, k, idx_out);
-  // k <= 32: the admission runs inside the saliency kernel; larger k takes
-  // the separate single-block selection
-  const bool fused = k > 0 && k <= kFusedMaxK;
+  // per head with k <= 32: the admission runs inside the saliency kernel;
+  // larger k, or the head-averaged selection, takes a kernel of its own
+  const bool fused = !shared && k > 0 && k <= kFusedMaxK;
   if ((s = attend_impl(h, layer, Q, K, V, out, saliency, fused ? &a : nullptr, sst)) != REGMEM_OK)
     return s;
   if (k > 0 && !fused) {
-    RM_CUDA(h, launch_admit(a, sst));
+    RM_CUDA(h, shared ? launch_admit_shared(a, sst) : launch_admit(a, sst));
     h->prof.launches_admit += 1;
   }
   h->len[layer] += k;
   return finish_side(h, layer, sst);
+}
+
+}  // namespace
+
+regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const void* Q, const void* K,
+                                  const void* V, void* out, float* saliency, int32_t k,
+                                  int32_t* idx_out) {
+  REGMEM_RANGE;
+  return attend_admit_impl(h, layer, Q, K, V, out, saliency, k, idx_out, false);
+}
+
+regmem_status regmem_attend_admit_shared(regmem_t* h, int32_t layer, const void* Q, const void* K,
+                                         const void* V, void* out, float* saliency, int32_t k,
+                                         int32_t* idx_out) {
+  REGMEM_RANGE;
+  return attend_admit_impl(h, layer, Q, K, V, out, saliency, k, idx_out, true);
 }
 
 namespace {

@@ -33,6 +33,7 @@ _SIGNATURES = {
     "regmem_admit": (ctypes.c_int, [_P, _I32, _I32, _P]),
     "regmem_admit_shared": (ctypes.c_int, [_P, _I32, _I32, _P]),
     "regmem_attend_admit": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, _I32, _P]),
+    "regmem_attend_admit_shared": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, _I32, _P]),
     "regmem_attend_admit_host": (ctypes.c_int, [_P, _I32, _P, _P, _P, _P, _P, _I32]),
     "regmem_frame_attention": (ctypes.c_int, [_P, _P, _P, _P, _P]),
     "regmem_reset": (ctypes.c_int, [_P]),
@@ -189,6 +190,11 @@ def regmem_attend_admit(h, layer, Q, K, V, out, saliency, k, idx_out=None):
                                                 _ptr(saliency), k, _ptr(idx_out)))
 
 
+def regmem_attend_admit_shared(h, layer, Q, K, V, out, saliency, k, idx_out=None):
+    return _check(h, load().regmem_attend_admit_shared(h, layer, _ptr(Q), _ptr(K), _ptr(V), _ptr(out),
+                                                       _ptr(saliency), k, _ptr(idx_out)))
+
+
 def regmem_attend_admit_host(h, layer, Q, K, V, out, saliency, k):
     return _check(h, load().regmem_attend_admit_host(h, layer, _ptr(Q), _ptr(K), _ptr(V),
                                                      _ptr(out), _ptr(saliency), k))
@@ -309,6 +315,10 @@ class RegMem:
 
     def attend_admit(self, layer, Q, K, V, out, saliency, k, idx_out=None):
         return regmem_attend_admit(self.h, layer, Q, K, V, out, saliency, k, idx_out)
+
+    def attend_admit_shared(self, layer, Q, K, V, out, saliency, k, idx_out=None):
+        """attend_frame + admit_shared in one call (side stream with overlap)."""
+        return regmem_attend_admit_shared(self.h, layer, Q, K, V, out, saliency, k, idx_out)
 
     def attend_admit_host(self, layer, Q, K, V, out, saliency, k):
         return regmem_attend_admit_host(self.h, layer, Q, K, V, out, saliency, k)

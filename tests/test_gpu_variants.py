@@ -71,6 +71,43 @@ def test_shared_admission_matches_oracle(kk):
         st.close()
 
 
+@pytest.mark.parametrize("overlap", [0, 1])
+def test_one_call_shared_admission_matches_two_calls(overlap):
+    """regmem_attend_admit_shared (saliency and head-averaged selection on the
+    side stream when overlap is on) against regmem_attend_frame +
+    regmem_admit_shared on another handle: O, saliency, the chosen tokens and
+    every layer's bank bit for bit, over the anchor and four admitted frames of
+    two layers."""
+    H, ns, gh, gw, kk = 16, 5, 37, 37, 14
+    N = ns + gh * gw
+    a = Stream(2, H, ns, gh, gw, budget=kk, max_frames=6, seed=35)
+    b = Stream(2, H, ns, gh, gw, budget=kk, max_frames=6, seed=35)
+    try:
+        a.rm.set_overlap(overlap)
+        for t in range(1, 6):
+            for l in range(2):
+                q, k, v = a.inputs(l, t)
+                oa, sa = torch.empty_like(q), torch.empty(H, N, dtype=torch.float32, device=q.device)
+                ia = torch.full((kk,), -1, dtype=torch.int32, device="cuda")
+                a.rm.attend_admit_shared(l, q, k, v, oa, sa, kk, ia)
+                ob, sb, _ = b.attend(l, q, k, v)
+                ib = torch.full((kk,), -1, dtype=torch.int32, device="cuda")
+                b.rm.admit_shared(l, kk, ib)
+                a.rm.synchronize()
+                b.rm.synchronize()
+                assert torch.equal(oa, ob) and torch.equal(sa, sb), (t, l)
+                if t > 1:
+                    assert torch.equal(ia, ib), (t, l)
+                assert a.rm.memory_len(l) == b.rm.memory_len(l) == N + (t - 1) * kk
+        for l in range(2):
+            ka, va = a.export(l)
+            kb, vb = b.export(l)
+            assert torch.equal(ka, kb) and torch.equal(va, vb)
+    finally:
+        a.close()
+        b.close()
+
+
 @pytest.mark.parametrize("H,ns,gh,gw,frames", [(2, 5, 8, 8, 6), (16, 5, 37, 37, 3)])
 def test_unregulated_full_kv_stream(H, ns, gh, gw, frames):
     """The full-KV memory: candidates = all tokens and k = N keep every frame
