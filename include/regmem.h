@@ -197,11 +197,14 @@ REGMEM_API regmem_status regmem_attend_admit(regmem_t* h, int32_t layer, const v
 
 /* regmem_attend_frame followed by regmem_admit_shared(layer, k, idx_out), in
  * one call: the per-frame step of one layer with the selection that keeps no
- * head-specific retention (Table 4, first row).  The saliency and the shared
- * selection run on the stream regmem_attend_admit uses for its side work (the
- * side stream when overlap is on).  Results are bit-identical to the two calls;
- * idx_out is an optional device int32 [k].  Arguments, checks, state and
- * validity of K, V and saliency as in regmem_attend_admit. */
+ * head-specific retention (Table 4, first row).  For k <= 32 the selection
+ * runs inside the saliency kernel: the last head to finish a key tile ranks
+ * the tile's head-summed saliency, and the last tile merges the lists and
+ * appends.  Larger k takes the separate selection kernel.  Both run on the
+ * stream regmem_attend_admit uses for its side work (the side stream when
+ * overlap is on).  Results are bit-identical to the two calls; idx_out is an
+ * optional device int32 [k].  Arguments, checks, state and validity of K, V
+ * and saliency as in regmem_attend_admit. */
 REGMEM_API regmem_status regmem_attend_admit_shared(regmem_t* h, int32_t layer, const void* Q,
                                          const void* K, const void* V, void* out,
                                          float* saliency, int32_t k, int32_t* idx_out);

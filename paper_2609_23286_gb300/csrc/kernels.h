@@ -256,11 +256,13 @@ struct AdmitArgs {
   int N, H, cand_lo, k;
   int32_t* idx_out;         // optional [H][k]
   // distributed selection (k <= 32): per-(head, 128-key tile) lists and
-  // per-head completion counters (zero between launches); null -> one block
-  // per head selects alone
+  // completion counters (zero between launches): per head, or with `shared`
+  // per key tile plus one for the tiles; null -> one block per head selects
+  // alone
   uint64_t* lists;          // [H][ceil(N/128)][32]
-  int* done;                // [H]
+  int* done;                // [max(H, ceil(N/128) + 1)]
   int* status;              // device status word (range guards of the checked build)
+  int shared;               // fused path only: one token set for all heads (idx_out [k])
 };
 cudaError_t admit_setup();
 // Per-head admission (Eq. 6): k rows per head, idx_out [H][k].

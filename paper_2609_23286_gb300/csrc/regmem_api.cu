@@ -74,7 +74,7 @@ struct regmem {
   int* qidx = nullptr;        // [nq]
   __nv_bfloat16* part_o = nullptr;  // split-KV partials
   float* part_lse = nullptr;
-  int* head_done = nullptr;   // per-head completion counters of the distributed selection
+  int* head_done = nullptr;   // completion counters of the distributed selection (per head or per key tile)
   // the attention's launch clock: kClockSlots start words, then as many end
   // words, one pair per launch since regmem_profile_enable
   unsigned long long* kclock = nullptr;
@@ -462,8 +462,11 @@ regmem_status regmem_set_frame(regmem_t* h, const regmem_frame_desc* fd) {
   RM_CUDA(h, cudaMemcpy(h->qidx, q.data(), q.size() * sizeof(int), cudaMemcpyHostToDevice));
   RM_CUDA(h, cudaMalloc(&h->part_o, attn_part_o_elems(h->attn_grid, kAttnMaxPhases) * sizeof(__nv_bfloat16)));
   RM_CUDA(h, cudaMalloc(&h->part_lse, attn_part_lse_floats(h->attn_grid, kAttnMaxPhases) * sizeof(float)));
-  RM_CUDA(h, cudaMalloc(&h->head_done, h->heads * sizeof(int)));
-  RM_CUDA(h, cudaMemset(h->head_done, 0, h->heads * sizeof(int)));
+  {  // per-head counters, or per key tile plus one (the shared selection)
+    const size_t nd = std::max(h->heads, (N + kTile - 1) / kTile + 1);
+    RM_CUDA(h, cudaMalloc(&h->head_done, nd * sizeof(int)));
+    RM_CUDA(h, cudaMemset(h->head_done, 0, nd * sizeof(int)));
+  }
   RM_CUDA(h, cudaMalloc(&h->adm_lists, (size_t)h->heads * ((N + kTile - 1) / kTile) * 32 * sizeof(uint64_t)));
   RM_CUDA(h, cudaHostAlloc(&h->status_host, sizeof(int), cudaHostAllocMapped));
   *h->status_host = 0;
@@ -673,10 +676,11 @@ regmem_status attend_admit_impl(regmem_t* h, int32_t layer, const void* Q, const
     return finish_side(h, layer, sst);
   }
   if ((s = check_admit(h, layer, k)) != REGMEM_OK) return s;
-  const AdmitArgs a = admit_args(h, layer, K, V, saliency, k, idx_out);
-  // per head with k <= 32: the admission runs inside the saliency kernel;
-  // larger k, or the head-averaged selection, takes a kernel of its own
-  const bool fused = !shared && k > 0 && k <= kFusedMaxK;
+  AdmitArgs a = admit_args(h, layer, K, V, saliency, k, idx_out);
+  a.shared = shared ? 1 : 0;
+  // k <= 32: the admission (per head, or head-averaged) runs inside the
+  // saliency kernel; larger k takes a selection kernel of its own
+  const bool fused = k > 0 && k <= kFusedMaxK;
   if ((s = attend_impl(h, layer, Q, K, V, out, saliency, fused ? &a : nullptr, sst)) != REGMEM_OK)
     return s;
   if (k > 0 && !fused) {

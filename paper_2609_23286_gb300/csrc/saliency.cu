@@ -22,7 +22,10 @@
 // block sorts its tile's candidates (select.cuh) and stores its best 32, then
 // adds itself to its head's completion counter; the last block of a head
 // merges the tiles' lists into the head's k admitted tokens, appends their K
-// and V rows to the bank and clears the counter for the next launch.
+// and V rows to the bank and clears the counter for the next launch.  With
+// `shared` (no head-specific retention) the counters are per key tile: the
+// last head of a tile ranks the head sums of its tokens, and the last tile
+// merges the lists and appends the same rows to every head.
 
 #include "kernels.h"
 #include "ptx.cuh"
@@ -234,10 +237,67 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
   }
   if (tid == 0 && sm.abort_flag) atomicOr(p.status, kStatusTimeout);
   if (p.adm_k < 1) return;
-  // ---- fused admission: this tile's best candidates, then the head's last
-  // block merges the tiles' lists and appends
   const bool cand = j < p.N && j >= p.adm.cand_lo;
   uint64_t* lists = reinterpret_cast<uint64_t*>(&sm.qs[0][0]);  // THREADS values
+  if (p.adm.shared) {
+    // ---- fused admission without head-specific retention (Table 4): the
+    // last head to finish a key tile ranks the tile's tokens by their
+    // saliency summed over the heads (heads added in ascending order, as the
+    // separate selection sums them); the last tile to finish merges the
+    // tiles' lists, and every head's bank receives the same k rows
+    __threadfence();  // this head's saliency before the tile's count
+    __syncthreads();
+    if (tid == 0) sm.last = atomicAdd(p.adm.done + kt, 1) == p.H - 1;
+    __syncthreads();
+    if (!sm.last) return;
+    __threadfence();
+    float sum = 0.f;
+    if (cand)
+      for (int hh = 0; hh < p.H; ++hh) sum += __ldcg(p.sal + (size_t)hh * p.N + j);
+    sel::block_top_list<THREADS>(cand ? sel::pack_candidate(sum, j) : 0ull, lists,
+                                 p.adm.lists + (size_t)kt * sel::kListK);
+    __threadfence();  // the list before the count
+    __syncthreads();
+    if (tid == 0) {
+      p.adm.done[kt] = 0;  // every head of this tile has counted
+      sm.last = atomicAdd(p.adm.done + nkt, 1) == nkt - 1;
+    }
+    __syncthreads();
+    if (!sm.last) return;
+    __threadfence();
+    int* ord = reinterpret_cast<int*>(&sm.qs[1][0]);
+    sel::merge_head_lists<THREADS>(p.adm.lists, nkt, p.adm_k, p.adm.cand_lo, lists, ord);
+    // every head's rows of the k tokens: 16-byte pieces (head, K or V, row,
+    // piece), eight loads in flight per thread before their stores
+    const int per_head = p.adm_k * 16, total = p.H * per_head;
+    for (int w0 = tid; w0 < total; w0 += THREADS * 8) {
+      uint4 v[8];
+      uint4* dst[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int w = w0 + u * THREADS;
+        dst[u] = nullptr;
+        if (w >= total) continue;
+        const int hh = w / per_head, rem = w - hh * per_head;
+        const int which = rem / (p.adm_k * 8), r = (rem >> 3) % p.adm_k, c = rem & 7;
+        const int tok = p.adm.cand_lo + ord[r];
+        if (!dev_check(tok >= p.adm.cand_lo && tok < p.N && p.adm.M + r < p.adm.cap, p.status)) continue;
+        const __nv_bfloat16* src = (which ? p.adm.V : p.adm.K) + ((size_t)tok * p.H + hh) * HD;
+        dst[u] = reinterpret_cast<uint4*>((which ? p.adm.bankV : p.adm.bankK) +
+                                          ((size_t)hh * p.adm.cap + p.adm.M + r) * HD) + c;
+        v[u] = reinterpret_cast<const uint4*>(src)[c];
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (dst[u]) *dst[u] = v[u];
+    }
+    if (p.adm.idx_out)
+      for (int r = tid; r < p.adm_k; r += THREADS) p.adm.idx_out[r] = p.adm.cand_lo + ord[r];
+    if (tid == 0) p.adm.done[nkt] = 0;
+    return;
+  }
+  // ---- fused admission: this tile's best candidates, then the head's last
+  // block merges the tiles' lists and appends
   sel::block_top_list<THREADS>(cand ? sel::pack_candidate(acc, j) : 0ull, lists,
                                p.adm.lists + ((size_t)h * nkt + kt) * sel::kListK);
   __threadfence();  // the list before the count
