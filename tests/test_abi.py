@@ -62,6 +62,8 @@ def test_host_side_validation_without_gpu(lib_path):
         assert lib.regmem_attend_frame(handle, 0, 16, 16, 16, 16, 16) == regmem.ERR_STATE
         assert "set_frame" in regmem.regmem_last_error(handle)
         assert lib.regmem_admit(handle, 0, 1, None) == regmem.ERR_STATE
+        for call in (lib.regmem_attend_admit, lib.regmem_attend_admit_shared):
+            assert call(handle, 0, 16, 16, 16, 16, 16, 1, None) == regmem.ERR_STATE  # before set_frame
         assert regmem.regmem_memory_len(handle, 1) == 0
         with pytest.raises(regmem.RegmemError):
             regmem.regmem_memory_len(handle, 2)
@@ -77,6 +79,7 @@ def test_host_side_validation_without_gpu(lib_path):
     assert lib.regmem_reset(None) == regmem.ERR_ARG
     assert lib.regmem_set_overlap(None, 1) == regmem.ERR_ARG
     assert lib.regmem_join(None) == regmem.ERR_ARG
+    assert lib.regmem_attend_admit_shared(None, 0, 16, 16, 16, 16, 16, 1, None) == regmem.ERR_ARG
 
 
 def _c_struct_fields(name):
