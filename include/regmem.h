@@ -167,7 +167,7 @@ REGMEM_API regmem_status regmem_attend_frame_host(regmem_t* h, int32_t layer, co
  * State: the layer must have an attend pending (ERR_STATE). */
 REGMEM_API regmem_status regmem_admit(regmem_t* h, int32_t layer, int32_t k, int32_t* idx_out);
 
-/* Admission without head-specific retention (the ablation of Sec. 4.3,
+/* Admission without head-specific retention (the ablation of Sec. 4.5,
  * Table 4, "w/o Head-specific Retention"): instead of each head ranking its
  * own saliency, one set of k candidate tokens is chosen for all heads, ranked
  * by the saliency summed over heads (fp32, heads added in ascending order;

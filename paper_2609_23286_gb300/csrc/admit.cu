@@ -10,7 +10,7 @@
 //   select.cuh over all of the head's candidates.
 //
 // admit_shared_kernel (any k): the selection without head-specific
-//   retention (the ablation of Sec. 4.3, Table 4): one index set for all heads,
+//   retention (the ablation of Sec. 4.5, Table 4): one index set for all heads,
 //   ranked by the head sum of the saliency (equivalently its head mean).
 //
 // copy_rows_kernel: rows [lo, lo + n) of the frame appended after row M of
