@@ -22,7 +22,7 @@ What it computes, per frame t, layer l and head h (paper notation):
   ``|M_t| = |M_1| + (t - 1) k``, with ``k = floor(gamma N)`` on the layers
   that admit (Eq. 6) and k = 0 on the anchor-only layers (Eq. 5); Sec. 4.1
   makes layers 11-17 (1-based) the admitting ones.
-* The selection without head-specific retention (the ablation of Sec. 4.3,
+* The selection without head-specific retention (the ablation of Sec. 4.5,
   Table 4): one set of k tokens for all heads, ranked by the saliency
   averaged over heads.
 * The unregulated stream (the full-KV memory the paper compares against):
@@ -153,7 +153,7 @@ def topk_admission(s: np.ndarray, n_special: int, k: int,
 
 def topk_admission_shared(s: np.ndarray, n_special: int, k: int,
                           candidates: str = "patch") -> list[int]:
-    """Top-k without head-specific retention (Sec. 4.3, Table 4, first row):
+    """Top-k without head-specific retention (Sec. 4.5, Table 4, first row):
     the saliency of all heads ``s`` [H, N] is averaged over heads and one set
     of k tokens is chosen for every head, ordered and tie-broken as in
     ``topk_admission``."""

@@ -1,7 +1,7 @@
 """Parity of the variants the paper studies around its default configuration,
 through the C ABI against the fp64 oracle:
 
-* selection without head-specific retention (Sec. 4.3, Table 4):
+* selection without head-specific retention (Sec. 4.5, Table 4):
   regmem_admit_shared;
 * the unregulated full-KV memory the paper compares against (every frame's
   N rows kept; candidates = all tokens, k = N);

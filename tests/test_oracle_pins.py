@@ -257,7 +257,7 @@ def check_permutation(mod):
 
 
 def check_shared_topk(mod):
-    """Selection without head-specific retention (Sec. 4.3, Table 4): the
+    """Selection without head-specific retention (Sec. 4.5, Table 4): the
     chosen set equals the rank-based top-k of the plain head average written
     out in Python (ties included); with one head it is the per-head choice;
     and on a crafted case where each head prefers a different token, the
