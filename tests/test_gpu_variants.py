@@ -71,14 +71,15 @@ def test_shared_admission_matches_oracle(kk):
         st.close()
 
 
-@pytest.mark.parametrize("overlap", [0, 1])
-def test_one_call_shared_admission_matches_two_calls(overlap):
+@pytest.mark.parametrize("overlap,kk", [(0, 14), (1, 14), (1, 1), (1, 32), (1, 33)])
+def test_one_call_shared_admission_matches_two_calls(overlap, kk):
     """regmem_attend_admit_shared (saliency and head-averaged selection on the
-    side stream when overlap is on) against regmem_attend_frame +
+    side stream when overlap is on; fused into the saliency kernel for k <= 32,
+    the separate selection kernel above) against regmem_attend_frame +
     regmem_admit_shared on another handle: O, saliency, the chosen tokens and
     every layer's bank bit for bit, over the anchor and four admitted frames of
     two layers."""
-    H, ns, gh, gw, kk = 16, 5, 37, 37, 14
+    H, ns, gh, gw = 16, 5, 37, 37
     N = ns + gh * gw
     a = Stream(2, H, ns, gh, gw, budget=kk, max_frames=6, seed=35)
     b = Stream(2, H, ns, gh, gw, budget=kk, max_frames=6, seed=35)
