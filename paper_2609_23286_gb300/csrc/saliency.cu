@@ -122,6 +122,9 @@ __device__ __forceinline__ void gather_lse(const Params& p, int h, int g0, int g
     if (g0 + c < g1) sm.lse2[(g0 + c) % QS][tid] = tok[c] >= 0 ? lv[c] * 1.4426950408889634f : INFINITY;
 }
 
+// SHARED: the fused admission without head-specific retention (its own
+// instantiation, so the per-head kernel's code is unchanged by it).
+template <bool SHARED>
 __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant__ CUtensorMap tmK,
                                                            const Params p) {
   extern __shared__ uint8_t smem_raw[];
@@ -239,7 +242,7 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
   if (p.adm_k < 1) return;
   const bool cand = j < p.N && j >= p.adm.cand_lo;
   uint64_t* lists = reinterpret_cast<uint64_t*>(&sm.qs[0][0]);  // THREADS values
-  if (p.adm.shared) {
+  if constexpr (SHARED) {
     // ---- fused admission without head-specific retention (Table 4): the
     // last head to finish a key tile ranks the tile's tokens by their
     // saliency summed over the heads (heads added in ascending order, as the
@@ -316,7 +319,10 @@ __global__ void __launch_bounds__(THREADS) saliency_kernel(const __grid_constant
 }  // namespace
 
 cudaError_t saliency_setup() {
-  return cudaFuncSetAttribute(saliency_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  const cudaError_t e = cudaFuncSetAttribute(saliency_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(saliency_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)SMEM_BYTES);
 }
 
@@ -342,7 +348,9 @@ cudaError_t launch_saliency(const SalArgs& a, cudaStream_t s) {
     p.adm_k = a.adm->k;
   }
   const int nkt = (a.N + BT - 1) / BT;
-  return launch_pdl(saliency_kernel, dim3(a.H * nkt), dim3(THREADS), SMEM_BYTES, s, *a.tmK, p);
+  if (p.adm_k >= 1 && p.adm.shared)
+    return launch_pdl(saliency_kernel<true>, dim3(a.H * nkt), dim3(THREADS), SMEM_BYTES, s, *a.tmK, p);
+  return launch_pdl(saliency_kernel<false>, dim3(a.H * nkt), dim3(THREADS), SMEM_BYTES, s, *a.tmK, p);
 }
 
 }  // namespace regmem_dev
