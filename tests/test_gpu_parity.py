@@ -66,6 +66,17 @@ def test_tiny_stream_full_oracle(fused):
     run_stream(1, 2, 5, 8, 8, 1, 8, seed=0, fused=fused)
 
 
+@pytest.mark.parametrize("fused", [False, True])
+@pytest.mark.parametrize("H,ns,gh,gw", [(1, 0, 1, 1), (3, 1, 1, 2), (2, 0, 3, 1)])
+def test_degenerate_frames(H, ns, gh, gw, fused):
+    """The smallest frames: one token (no special tokens, a 1 x 1 patch grid:
+    one sampled query, one admission candidate), three tokens (one special,
+    1 x 2 patches) and a 3 x 1 grid.  Every query and key tile is a single
+    ragged row or a few; the stream admits one row per frame, against the
+    oracle frame by frame."""
+    run_stream(1, H, ns, gh, gw, 1, 5, seed=H * 10 + gh, fused=fused)
+
+
 @pytest.mark.parametrize("ds", [1, 3, 4])
 def test_query_downsampling_factors(ds):
     """Sec. 3.3 with other windows (T6's sweep): 13 x 11 patches + 5 specials,
