@@ -77,6 +77,15 @@ def test_degenerate_frames(H, ns, gh, gw, fused):
     run_stream(1, H, ns, gh, gw, 1, 5, seed=H * 10 + gh, fused=fused)
 
 
+@pytest.mark.parametrize("k,fused", [(14, True), (40, False)])
+def test_largest_candidate_set(k, fused):
+    """Frames at the library's limit of admission candidates: 2 special tokens
+    and 90 x 91 patches (N = 8,192, 8,190 candidates, 2,116 sampled queries):
+    the fused selection over 64 key tiles' lists (k = 14) and the radix
+    selection of the two-call path (k = 40), against the full oracle."""
+    run_stream(1, 2, 2, 90, 91, k, 2, seed=77 + k, fused=fused)
+
+
 @pytest.mark.parametrize("ds", [1, 3, 4])
 def test_query_downsampling_factors(ds):
     """Sec. 3.3 with other windows (T6's sweep): 13 x 11 patches + 5 specials,
